@@ -1,0 +1,421 @@
+/*
+ * isjl_oracle.c -- CPU oracle for the batched FCFS / LJF / ISJL simulator.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the plain, slow, step-by-step
+ * statement of what the scheduling model of "Efficiency and Cost Alignment in
+ * Batched LLM Serving via Resource-Fair Scheduling" computes.  Only the tests,
+ * the package's smoke check and the benchmark's CPU-baseline leg may load it.
+ * It shares no code, header, table or helper with the CUDA path.
+ *
+ * Model (Section 2, "Model"): request i needs o_i = prompt_i + output_i
+ * tokens, processed one token per step; at most B requests run in a step;
+ * progress a_i is the KV footprint; the fairness constraint (Eq. 1) bounds
+ * max a - min a over the running set by the budget alpha (called delta here).
+ * Service is contiguous: a started request runs every step until done
+ * (integer program of Appendix A, constraint (2)).
+ *
+ * Cost (Section 5, Eq. batch-cost-progress): a nonempty step costs
+ * c + tau*|S|*max r with r_i = a_i + 1.  Decomposition (Theorem "Profit
+ * decomposition"): total = tau*Q + c*T + tau*E with Q = sum o(o+1)/2 and
+ * E = sum over steps of sum_{i in S}(max r - r_i).
+ *
+ * Readings where the paper is silent (each is listed in the design notes):
+ *   - KV cap: a running request reserves its peak footprint o_i; a start needs
+ *     sum_{S} o_j + o_i <= kv_cap.  kv_cap = INT32_MAX is the paper's model.
+ *   - In every policy the first KV failure ends all starts of that step.
+ *   - "Longest" = (o descending, index ascending); arrival order = index order.
+ *   - A request started in step k runs in step k; completion c_i = (last step
+ *     it ran) + 1; T_busy counts nonempty steps, T_make = max c_i.
+ *   - ISJL: see isjl_admit() below.
+ */
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define OR_FCFS 0
+#define OR_LJF  1
+#define OR_ISJL 2
+
+#define OR_OK            0
+#define OR_INVALID_ARG   1
+#define OR_INFEASIBLE    2
+#define OR_OOM           3
+#define OR_STEP_LIMIT    5
+
+#define ST_WAIT    0   /* not started, not in a plan (released or not) */
+#define ST_PLANNED 1   /* placed in an ISJL Phase ONE plan, not started */
+#define ST_RUN     2
+#define ST_DONE    3
+
+typedef struct {
+    int64_t T_make, T_busy, O, Q, W, E, token_adv;
+    int64_t sum_completion, sum_latency, sum_extent, max_extent;
+    int64_t violations, kv_violations, peak_kv, peak_batch, status;
+    double c_T, tau_Q, tau_E, cost, revenue, profit, throughput, ael;
+} or_record;
+
+typedef struct {
+    int n, B, policy;
+    int64_t alpha, kv_cap;
+    const int32_t *arr;
+    int32_t *o;
+    int32_t *status, *a, *start, *compl;
+    int32_t *by_len;          /* job ids sorted by (o desc, idx asc) */
+    /* running set */
+    int32_t *run;  int run_cnt;  int64_t kv_sum;
+    /* FCFS */
+    int next_fcfs;
+    /* ISJL workers, 1-based: worker_job[j] running job or -1; plan FIFO */
+    int32_t *worker_job, *plan_head, *plan_tail, *plan_next, *job_worker;
+    int64_t plan_left;
+    int64_t t0, d1;
+    int32_t L1;               /* o_1 of the current stage (worker 1) */
+    int32_t *long_of;         /* long_of[j]: o_j planned on worker j, 2..M */
+} sim_t;
+
+/* ---- sorting by (o desc, idx asc) --------------------------------------- */
+static const int32_t *g_sort_o;
+static int cmp_len(const void *x, const void *y) {
+    int32_t i = *(const int32_t *)x, j = *(const int32_t *)y;
+    if (g_sort_o[i] != g_sort_o[j]) return g_sort_o[i] > g_sort_o[j] ? -1 : 1;
+    return i < j ? -1 : (i > j);
+}
+
+static int64_t min64(int64_t x, int64_t y) { return x < y ? x : y; }
+static int64_t max64(int64_t x, int64_t y) { return x > y ? x : y; }
+
+/* ---- common start / helpers ---------------------------------------------- */
+static void start_job(sim_t *s, int32_t i, int64_t k, int worker) {
+    s->status[i] = ST_RUN;
+    s->a[i] = 0;
+    s->start[i] = (int32_t)k;
+    s->run[s->run_cnt++] = i;
+    s->kv_sum += s->o[i];
+    if (s->policy == OR_ISJL) { s->worker_job[worker] = i; s->job_worker[i] = worker; }
+}
+
+/* longest released request that is neither running, done nor planned */
+static int32_t longest_waiting(const sim_t *s, int64_t k) {
+    for (int p = 0; p < s->n; ++p) {
+        int32_t i = s->by_len[p];
+        if (s->status[i] == ST_WAIT && s->arr[i] <= k) return i;
+    }
+    return -1;
+}
+
+/* A_max(k): largest progress among running requests (0 when none run) */
+static int64_t a_max(const sim_t *s) {
+    int64_t m = 0;
+    for (int q = 0; q < s->run_cnt; ++q) m = max64(m, s->a[s->run[q]]);
+    return m;
+}
+
+/* ---- FCFS (Section 2.1 example, continuous-batching remark) -------------- */
+/* Each step admit released requests in arrival (= index) order while a slot
+ * is free and the KV reservation fits; the first request that does not fit
+ * ends admissions, so requests never overtake each other.  FCFS ignores the
+ * fairness budget: it is the unconstrained baseline. */
+static void fcfs_admit(sim_t *s, int64_t k) {
+    while (s->run_cnt < s->B && s->next_fcfs < s->n && s->arr[s->next_fcfs] <= k) {
+        int32_t i = s->next_fcfs;
+        if (s->kv_sum + s->o[i] > s->kv_cap) break;
+        start_job(s, i, k, 0);
+        s->next_fcfs++;
+    }
+}
+
+/* ---- LJF (Algorithm 1, static batching remark) -------------------------- */
+/* When nothing runs, form a batch of the longest released requests (at most
+ * B, stopping at the first KV failure) and hold it until every member is
+ * done.  Offline with no KV cap this is exactly Algorithm 1's consecutive
+ * groups o_1..o_B, o_{B+1}..o_{2B}, ... */
+static void ljf_admit(sim_t *s, int64_t k) {
+    if (s->run_cnt != 0) return;
+    while (s->run_cnt < s->B) {
+        int32_t i = longest_waiting(s, k);
+        if (i < 0) break;
+        if (s->kv_sum + s->o[i] > s->kv_cap) break;
+        start_job(s, i, k, 0);
+    }
+}
+
+/* ---- ISJL (Algorithm 2 with beta = alpha; online rolling form, Sec. 3.4) - */
+static void plan_append(sim_t *s, int j, int32_t i) {
+    s->status[i] = ST_PLANNED;
+    s->plan_next[i] = -1;
+    if (s->plan_head[j] < 0) s->plan_head[j] = i; else s->plan_next[s->plan_tail[j]] = i;
+    s->plan_tail[j] = i;
+    s->plan_left++;
+}
+
+/* Phase ONE at a stage start (nothing runs, no plan entry is left, and the
+ * released queue Q(k) is nonempty).  Returns 1 if a plan was made. */
+static int isjl_phase_one(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_t *budget) {
+    const int64_t al = s->alpha;
+    int q = 0;
+    /* Q(k) in the order o_1 >= o_2 >= ... (ties: lower index first) */
+    for (int p = 0; p < s->n; ++p) {
+        int32_t i = s->by_len[p];
+        if (s->status[i] == ST_WAIT && s->arr[i] <= k) Q[q++] = i;
+    }
+    s->t0 = k;
+    s->d1 = 0;
+    s->L1 = -1;
+    /* |Q| = 1 or o_2 <= alpha: go straight to Phase TWO */
+    if (q < 2 || (int64_t)s->o[Q[1]] <= al) return 0;
+
+    /* M = min{B, #{o_i > alpha}}  (called n_long to avoid the KV-cap clash) */
+    int cnt_long = 0;
+    for (int p = 0; p < q; ++p) if ((int64_t)s->o[Q[p]] > al) cnt_long++;
+    int n_long = cnt_long < s->B ? cnt_long : s->B;
+    const int64_t o1 = s->o[Q[0]];
+    const int64_t theta = min64(2 * al, o1 - (int64_t)s->o[Q[n_long - 1]] + al);
+
+    /* packing budgets: workers 2..M get cap_j = min{2 alpha, o_1 - o_j + alpha},
+     * workers M+1..B get alpha */
+    for (int j = 1; j <= s->B; ++j) { packsum[j] = 0; budget[j] = -1; }
+    for (int j = 2; j <= n_long; ++j) budget[j] = min64(2 * al, o1 - (int64_t)s->o[Q[j - 1]] + al);
+    for (int j = n_long + 1; j <= s->B; ++j) budget[j] = al;
+
+    /* the long requests leave the queue (worker j will run o_j) */
+    for (int p = 0; p < n_long; ++p) s->status[Q[p]] = ST_PLANNED;
+
+    /* first fit of the short requests o_i <= theta that follow the long ones,
+     * in sorted order: workers M+1..B (budget alpha) first, then workers
+     * M, M-1, ..., 2 (budget cap_j).  A request that fits nowhere stays in Q. */
+    for (int p = n_long; p < q; ++p) {
+        int32_t i = Q[p];
+        int64_t oi = s->o[i];
+        if (oi > theta) continue;
+        int placed = 0;
+        for (int j = n_long + 1; j <= s->B && !placed; ++j)
+            if (oi + packsum[j] <= budget[j]) { plan_append(s, j, i); packsum[j] += oi; placed = 1; }
+        for (int j = n_long; j >= 2 && !placed; --j)
+            if (oi + packsum[j] <= budget[j]) { plan_append(s, j, i); packsum[j] += oi; placed = 1; }
+    }
+    /* worker 1 runs o_1; worker j in 2..M runs its pack, then o_j */
+    plan_append(s, 1, Q[0]);
+    s->L1 = Q[0];
+    for (int j = 0; j <= s->B; ++j) s->long_of[j] = -1;
+    for (int j = 2; j <= n_long; ++j) { plan_append(s, j, Q[j - 1]); s->long_of[j] = Q[j - 1]; }
+
+    /* o_1 waits d1 = min{max{max_j sum(w_j) - alpha, 0}, alpha} steps, j = 2..M */
+    int64_t mx = 0;
+    for (int j = 2; j <= n_long; ++j) mx = max64(mx, packsum[j]);
+    s->d1 = min64(max64(mx - al, 0), al);
+    return 1;
+}
+
+/* ISJL admission for step k:
+ *   1. stage start (Phase ONE) when nothing runs, no plan entry is left and
+ *      Q(k) is nonempty;
+ *   2. plan starts, workers 1..B in order: an idle worker with plan entries
+ *      starts its next entry if A_max(k) <= alpha and the KV reservation fits;
+ *      worker 1's o_1 also waits until k >= t0 + d1 (waived once a later step
+ *      finds nothing running), and a long request o_j (j >= 2) also waits
+ *      until o_1 has started (Section 3.3: the pack tails run "in parallel
+ *      with o_1", and o_j follows its pack).  A blocked entry waits on its
+ *      worker;
+ *   3. Phase TWO: while a worker is free (not running, no plan entries), Q(k)
+ *      is nonempty and A_max(k) <= alpha, start the longest released request.
+ * Requests arriving during a stage only join Q(k) (never the current plan).
+ * A start always has progress 0, so A_max(k) is the same for every start of
+ * the step. */
+static void isjl_admit(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_t *budget) {
+    const int nothing_runs = (s->run_cnt == 0);
+    if (nothing_runs && s->plan_left == 0 && longest_waiting(s, k) >= 0)
+        isjl_phase_one(s, k, Q, packsum, budget);
+
+    const int gate_ok = a_max(s) <= s->alpha;
+    int stop = !gate_ok;
+
+    for (int j = 1; j <= s->B && !stop; ++j) {
+        int32_t e = s->plan_head[j];
+        if (e < 0 || s->worker_job[j] >= 0) continue;
+        if (j == 1 && e == s->L1) {
+            int delay_over = (k >= s->t0 + s->d1) || (k > s->t0 && nothing_runs);
+            if (!delay_over) continue;
+        }
+        if (j >= 2 && e == s->long_of[j] && s->status[s->L1] == ST_PLANNED) continue;
+        if (s->kv_sum + s->o[e] > s->kv_cap) { stop = 1; break; }
+        s->plan_head[j] = s->plan_next[e];
+        if (s->plan_head[j] < 0) s->plan_tail[j] = -1;
+        s->plan_left--;
+        start_job(s, e, k, j);
+    }
+    if (stop) return;
+
+    for (;;) {
+        int w = -1;
+        for (int j = 1; j <= s->B; ++j)
+            if (s->worker_job[j] < 0 && s->plan_head[j] < 0) { w = j; break; }
+        if (w < 0) break;
+        int32_t i = longest_waiting(s, k);
+        if (i < 0) break;
+        if (s->kv_sum + s->o[i] > s->kv_cap) break;
+        start_job(s, i, k, w);
+    }
+}
+
+/* ---- the run ------------------------------------------------------------- */
+/* Simulate one instance under one policy.  delta is the fairness budget
+ * (INT32_MAX = no constraint; ignored by FCFS and LJF except for counting
+ * violations).  start_out/compl_out may be NULL.  Returns the status. */
+int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
+               const int32_t *arrival, const int32_t *prompt, const int32_t *output,
+               double c, double tau, double p0, int64_t max_steps,
+               int32_t *start_out, int32_t *compl_out, or_record *rec)
+{
+    memset(rec, 0, sizeof(*rec));
+    if (n < 1 || B < 1 || delta < 0 || kv_cap < 1 || policy < 0 || policy > 2 || !arrival || !prompt || !output) {
+        rec->status = OR_INVALID_ARG; return OR_INVALID_ARG;
+    }
+    for (int i = 0; i < n; ++i) {
+        if (arrival[i] < 0 || prompt[i] < 0 || output[i] < 0 || (i > 0 && arrival[i] < arrival[i - 1])) {
+            rec->status = OR_INVALID_ARG; return OR_INVALID_ARG;
+        }
+    }
+    sim_t S; memset(&S, 0, sizeof(S));
+    sim_t *s = &S;
+    s->n = n; s->B = B; s->policy = policy; s->alpha = delta; s->kv_cap = kv_cap; s->arr = arrival;
+    s->o = malloc(sizeof(int32_t) * n);
+    s->status = malloc(sizeof(int32_t) * n);
+    s->a = malloc(sizeof(int32_t) * n);
+    s->start = malloc(sizeof(int32_t) * n);
+    s->compl = malloc(sizeof(int32_t) * n);
+    s->by_len = malloc(sizeof(int32_t) * n);
+    s->run = malloc(sizeof(int32_t) * (size_t)(B < n ? B : n) + sizeof(int32_t));
+    int32_t *Q = malloc(sizeof(int32_t) * n);
+    int64_t *packsum = malloc(sizeof(int64_t) * (size_t)(B + 1));
+    int64_t *budget = malloc(sizeof(int64_t) * (size_t)(B + 1));
+    s->worker_job = malloc(sizeof(int32_t) * (size_t)(B + 1));
+    s->plan_head = malloc(sizeof(int32_t) * (size_t)(B + 1));
+    s->plan_tail = malloc(sizeof(int32_t) * (size_t)(B + 1));
+    s->plan_next = malloc(sizeof(int32_t) * n);
+    s->job_worker = malloc(sizeof(int32_t) * n);
+    s->long_of = malloc(sizeof(int32_t) * (size_t)(B + 1));
+    int status = OR_OK;
+    if (!s->o || !s->status || !s->a || !s->start || !s->compl || !s->by_len || !s->run || !Q ||
+        !packsum || !budget || !s->worker_job || !s->plan_head || !s->plan_tail || !s->plan_next || !s->job_worker || !s->long_of) {
+        status = OR_OOM; goto done;
+    }
+
+    /* o_i = prompt + output (Section 2: prompt and output tokens, one per step) */
+    int64_t O = 0, Qsum = 0, sumA = 0, maxA = 0;
+    for (int i = 0; i < n; ++i) {
+        int64_t oi = (int64_t)prompt[i] + output[i];
+        if (oi < 1 || oi > kv_cap || oi > INT32_MAX / 2) { status = OR_INFEASIBLE; goto done; }
+        s->o[i] = (int32_t)oi;
+        O += oi;
+        Qsum += oi * (oi + 1) / 2;          /* Eq. intrinsic-resource-cost */
+        sumA += arrival[i];
+        if (arrival[i] > maxA) maxA = arrival[i];
+        s->status[i] = ST_WAIT; s->a[i] = 0; s->start[i] = -1; s->compl[i] = -1;
+        s->by_len[i] = i; s->plan_next[i] = -1; s->job_worker[i] = -1;
+    }
+    g_sort_o = s->o;
+    qsort(s->by_len, (size_t)n, sizeof(int32_t), cmp_len);
+    for (int j = 0; j <= B; ++j) {
+        s->worker_job[j] = -1; s->plan_head[j] = -1; s->plan_tail[j] = -1; s->long_of[j] = -1;
+    }
+    if (max_steps <= 0) max_steps = O + maxA + 1;
+
+    int done_cnt = 0;
+    int64_t W = 0, E = 0, T_busy = 0, tok = 0, sum_ext = 0, max_ext = 0, viol = 0, kv_viol = 0;
+    int64_t peak_kv = 0, peak_b = 0, T_make = 0, sum_c = 0;
+    for (int64_t k = 0;; ++k) {
+        if (k > max_steps) { status = OR_STEP_LIMIT; break; }
+        /* retire: requests whose progress reached o_i in step k-1 */
+        int w = 0;
+        for (int q = 0; q < s->run_cnt; ++q) {
+            int32_t i = s->run[q];
+            if (s->a[i] == s->o[i]) {
+                s->status[i] = ST_DONE;
+                s->compl[i] = (int32_t)k;
+                s->kv_sum -= s->o[i];
+                done_cnt++;
+                sum_c += k;
+                if (k > T_make) T_make = k;
+                if (policy == OR_ISJL) s->worker_job[s->job_worker[i]] = -1;
+            } else {
+                s->run[w++] = i;
+            }
+        }
+        s->run_cnt = w;
+        if (done_cnt == n) break;
+
+        /* admission */
+        if (policy == OR_FCFS) fcfs_admit(s, k);
+        else if (policy == OR_LJF) ljf_admit(s, k);
+        else isjl_admit(s, k, Q, packsum, budget);
+
+        /* serve step k: every running request processes token r_i = a_i + 1 */
+        if (s->run_cnt > 0) {
+            int64_t m = 0, mn = INT64_MAX, kvs = 0;
+            for (int q = 0; q < s->run_cnt; ++q) {
+                int64_t r = (int64_t)s->a[s->run[q]] + 1;
+                if (r > m) m = r;
+                if (r < mn) mn = r;
+                kvs += s->o[s->run[q]];
+            }
+            int64_t cnt = s->run_cnt;
+            W += cnt * m;                                   /* |S| * max r   */
+            for (int q = 0; q < s->run_cnt; ++q)            /* sum (max r - r_i) */
+                E += m - ((int64_t)s->a[s->run[q]] + 1);
+            int64_t ext = m - mn;                           /* Eq. 1 left side */
+            sum_ext += ext;
+            if (ext > max_ext) max_ext = ext;
+            if (ext > delta) viol++;
+            if (kvs > kv_cap) kv_viol++;
+            if (kvs > peak_kv) peak_kv = kvs;
+            if (cnt > peak_b) peak_b = cnt;
+            for (int q = 0; q < s->run_cnt; ++q) s->a[s->run[q]] += 1;
+            T_busy++;
+            tok += cnt;
+        }
+    }
+
+    rec->T_make = T_make; rec->T_busy = T_busy; rec->O = O; rec->Q = Qsum; rec->W = W; rec->E = E;
+    rec->token_adv = tok; rec->sum_completion = sum_c; rec->sum_latency = sum_c - sumA;
+    rec->sum_extent = sum_ext; rec->max_extent = max_ext; rec->violations = viol;
+    rec->kv_violations = kv_viol; rec->peak_kv = peak_kv; rec->peak_batch = peak_b;
+    /* cost decomposition C = tau Q + c T + tau E, profit = p0 O - C (Theorem
+     * "Profit decomposition"); evaluated in this order, without contraction */
+    rec->c_T = c * (double)T_busy;
+    rec->tau_Q = tau * (double)Qsum;
+    rec->tau_E = tau * (double)E;
+    rec->cost = (rec->c_T + rec->tau_Q) + rec->tau_E;
+    rec->revenue = p0 * (double)O;
+    rec->profit = rec->revenue - rec->cost;
+    rec->throughput = T_make > 0 ? (double)O / (double)T_make : 0.0;
+    rec->ael = (double)sum_c / (double)n;
+    if (start_out) memcpy(start_out, s->start, sizeof(int32_t) * n);
+    if (compl_out) memcpy(compl_out, s->compl, sizeof(int32_t) * n);
+done:
+    rec->status = status;
+    free(s->o); free(s->status); free(s->a); free(s->start); free(s->compl); free(s->by_len);
+    free(s->run); free(Q); free(packsum); free(budget); free(s->worker_job); free(s->plan_head);
+    free(s->plan_tail); free(s->plan_next); free(s->job_worker); free(s->long_of);
+    return status;
+}
+
+/* Run many instances (row-major, n per row) under one (policy, delta).
+ * rec has n_inst entries; start_out/compl_out are n_inst*n or NULL.
+ * Returns the first nonzero status, else 0. */
+int oracle_run_batch(int policy, int B, int64_t delta, int64_t kv_cap, int n_inst, int n,
+                     const int32_t *arrival, const int32_t *prompt, const int32_t *output,
+                     double c, double tau, double p0, int64_t max_steps,
+                     int32_t *start_out, int32_t *compl_out, or_record *rec)
+{
+    int first = 0;
+    for (int t = 0; t < n_inst; ++t) {
+        size_t off = (size_t)t * (size_t)n;
+        int st = oracle_run(policy, B, delta, kv_cap, n, arrival + off, prompt + off, output + off,
+                            c, tau, p0, max_steps, start_out ? start_out + off : NULL,
+                            compl_out ? compl_out + off : NULL, rec + t);
+        if (st && !first) first = st;
+    }
+    return first;
+}
+
+int oracle_record_size(void) { return (int)sizeof(or_record); }

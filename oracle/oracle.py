@@ -1,0 +1,96 @@
+"""ctypes front end of the CPU oracle (test infrastructure only).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline
+leg may import this module.  It loads ``oracle/_build/liboracle.so`` (built by
+``oracle/build.py``) and exposes:
+
+  run(policy, B, delta, kv_cap, arrival, prompt, output, ...) -> (records, start, completion)
+  opt_makespan(arrival, o, B, delta, kv_cap) -> optimal makespan (tiny instances)
+
+``policy`` is "fcfs", "ljf" or "isjl".  Arrays are int32 of shape
+(n_instances, n) or (n,).  ``delta``/``kv_cap`` of INT32_MAX mean "no limit".
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+INT32_MAX = 2**31 - 1
+POLICIES = {"fcfs": 0, "ljf": 1, "isjl": 2}
+STATUS = {0: "ok", 1: "invalid_arg", 2: "infeasible", 3: "oom", 5: "step_limit"}
+
+RECORD_FIELDS_I64 = ["T_make", "T_busy", "O", "Q", "W", "E", "token_adv",
+                     "sum_completion", "sum_latency", "sum_extent", "max_extent",
+                     "violations", "kv_violations", "peak_kv", "peak_batch", "status"]
+RECORD_FIELDS_F64 = ["c_T", "tau_Q", "tau_E", "cost", "revenue", "profit", "throughput", "ael"]
+RECORD_DTYPE = np.dtype([(f, np.int64) for f in RECORD_FIELDS_I64] +
+                        [(f, np.float64) for f in RECORD_FIELDS_F64])
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        path = _build.build()
+        L = ctypes.CDLL(path)
+        p32 = ctypes.POINTER(ctypes.c_int32)
+        L.oracle_run_batch.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
+                                       ctypes.c_int, ctypes.c_int, p32, p32, p32,
+                                       ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                       ctypes.c_int64, p32, p32, ctypes.c_void_p]
+        L.oracle_run_batch.restype = ctypes.c_int
+        L.oracle_record_size.restype = ctypes.c_int
+        L.oracle_opt_makespan.argtypes = [ctypes.c_int, p32, p32, ctypes.c_int, ctypes.c_int64,
+                                          ctypes.c_int64, ctypes.c_int64]
+        L.oracle_opt_makespan.restype = ctypes.c_int64
+        if L.oracle_record_size() != RECORD_DTYPE.itemsize:
+            raise RuntimeError("oracle record layout mismatch")
+        _lib = L
+    return _lib
+
+
+def _i32(x):
+    return np.ascontiguousarray(np.asarray(x, dtype=np.int32))
+
+
+def _ptr(a):
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+
+
+def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p0=0.002,
+        max_steps=0, per_request=True):
+    """Simulate every instance (row) under one policy and budget.
+
+    Returns (records, start, completion); records is a structured array with
+    one entry per instance (fields RECORD_DTYPE), start/completion are int32
+    arrays shaped like ``arrival`` (None when per_request is False).
+    """
+    a, p, o = _i32(arrival), _i32(prompt), _i32(output)
+    squeeze = a.ndim == 1
+    if squeeze:
+        a, p, o = a[None], p[None], o[None]
+    n_inst, n = a.shape
+    rec = np.zeros(n_inst, RECORD_DTYPE)
+    st = np.full((n_inst, n), -1, np.int32) if per_request else None
+    co = np.full((n_inst, n), -1, np.int32) if per_request else None
+    lib().oracle_run_batch(POLICIES[policy], int(B), int(delta), int(kv_cap), n_inst, n,
+                           _ptr(a), _ptr(p), _ptr(o), float(c), float(tau), float(p0), int(max_steps),
+                           _ptr(st) if per_request else None, _ptr(co) if per_request else None,
+                           rec.ctypes.data)
+    if squeeze:
+        rec = rec[0]
+        st = st[0] if per_request else None
+        co = co[0] if per_request else None
+    return rec, st, co
+
+
+def opt_makespan(arrival, o, B, delta, kv_cap=INT32_MAX, max_T=100_000):
+    """Exact optimal makespan of one tiny instance (n <= 9, o_i <= 62)."""
+    a, oo = _i32(arrival), _i32(o)
+    return int(lib().oracle_opt_makespan(len(oo), _ptr(a), _ptr(oo), int(B), int(delta),
+                                         int(kv_cap), int(max_T)))

@@ -1,0 +1,52 @@
+"""ISJL against the exhaustive offline optimum on the tiny-exhaustive workload.
+
+Theorem "Competitive ratio of Algorithm ISJL" (B = 2) and Theorem "Competitive
+ratio of Algorithm 2" (B >= 2) claim T_OPT / T_ISJL >= 3/4 offline with no KV
+cap.  For B = 2 the oracle meets it, and the sharper CR(gamma) bound, on all
+4096 instances.  For B = 3 it misses both on the instances listed in
+tests/golden/cr_findings.txt (a finding about Algorithm 2's generalisation,
+recorded, not hidden); this test pins that exact list.
+"""
+import os
+import sys
+
+import pytest
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, os.path.join(HERE, "golden"))
+import make_cr_findings as F  # noqa: E402
+
+INF = 2**31 - 1
+
+
+def load_findings():
+    out = {}
+    for line in open(os.path.join(HERE, "golden", "cr_findings.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        B, d, bound, cnt, *ids = line.split()
+        d = INF if d == "inf" else int(d)
+        out[(int(B), d, bound)] = [int(x) for x in ids]
+        assert len(ids) == int(cnt)
+    return out
+
+
+@pytest.fixture(scope="module")
+def computed():
+    return F.compute()
+
+
+def test_b2_meets_three_quarters_and_gamma(computed):
+    for d in F.DELTAS:
+        f34, fg = computed[(2, d)]
+        assert f34 == [] and fg == [], (d, f34[:5], fg[:5])
+
+
+def test_b3_misses_match_recorded_findings(computed):
+    rec = load_findings()
+    for d in F.DELTAS:
+        f34, fg = computed[(3, d)]
+        assert f34 == rec[(3, d, "3/4")]
+        assert fg == rec[(3, d, "gamma")]
+    # the bound holds at both ends of the budget range
+    assert computed[(3, 0)] == ([], []) and computed[(3, INF)] == ([], [])
