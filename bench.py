@@ -1,0 +1,366 @@
+#!/usr/bin/env python
+"""Benchmark: simulated batch-steps per second of the online delta-sweep.
+
+One step = one sweep of the whole hot path (derive, sort, simulate,
+summarize) over the online delta-sweep workload: 10,000 instances x 1,000
+requests (Poisson arrivals, mean gap 2 steps; prompt lognormal(ln 512, 1)
+clipped [16, 4096]; output lognormal(ln 256, 1.2) clipped [1, 2048]), KV cap
+200,000 tokens, B = 256 batch slots, runs FCFS, LJF and ISJL at
+delta in {16, 64, 256, 1024, inf} (7 runs per instance), per-request start and
+completion steps written out.  A batch-step is a simulated step whose batch
+is nonempty; value = sum over (instance, run) of T_busy per second.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--kernel step|epoch]
+  python bench.py --impl reference ...     (the CPU oracle on host cores)
+
+Multi-GPU (torchrun): rank r simulates its own replica of the workload
+(independent instances, weak scaling, no collective on the data path); the
+timing is the max over ranks.  Prints one JSON line on rank 0.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import multiprocessing as mp
+import os
+import platform
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_02244_gb300 import workloads as W  # noqa: E402
+
+METRIC = "simulated batch-steps/sec on 1 GB300 (ISJL Δ-sweep); % of HBM/int roofline"
+UNIT = "batch-steps/s"
+WID = 3
+INF = W.DELTA_INF
+POLICIES = ["fcfs", "ljf", "isjl", "isjl", "isjl", "isjl", "isjl"]
+DELTAS = [0, 0, 16, 64, 256, 1024, INF]
+# int32 ALU lanes per SM on GB300 (4 SM sub-partitions x 32 lanes) and SM count
+ALU_LANES_PER_SM = 128
+# algorithmic integer work of the per-step kernel: per token-advance
+# (r = a + 1, store, max, min, add/compare) and per batch-step (W, E, extent,
+# violation, T_busy, token counter)
+OPS_PER_TOKEN_ADVANCE = 5
+OPS_PER_BATCH_STEP = 6
+# DRAM bytes (read + write) per launch of the simulation kernel, scaled from an
+# ncu capture of a 512-instance case of this workload; None until captured
+SIM_DRAM_BYTES_PER_LAUNCH = None
+
+
+def workload_config(kernel, wl, flush):
+    return {
+        "workload": f"online-delta-sweep: {wl.n_instances} instances x {wl.n_per_instance} requests, "
+                    "Poisson arrivals mean gap 2; prompt LN(ln512,1) [16,4096]; output LN(ln256,1.2) [1,2048]",
+        "B": wl.B[0], "kv_cap": wl.kv_caps[0], "policies": POLICIES,
+        "deltas": ["inf" if d == INF else d for d in DELTAS],
+        "runs_per_instance": len(POLICIES), "per_request_outputs": True,
+        "kernel": kernel, "l2": flush,
+    }
+
+
+# ---------------------------------------------------------------- clocks ----
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons while timing."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid=None):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+        if uuid:
+            cmd += ["-i", uuid]
+        try:
+            self.p = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.p.terminate()
+        try:
+            out, _ = self.p.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+            out, _ = self.p.communicate()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------ CPU oracle ----
+def _oracle_chunk(args):
+    """Worker: run the oracle on a block of instances; returns (sum T_busy, sum token_adv)."""
+    a, p, o, B, kv = args
+    sys.path.insert(0, ROOT)
+    from oracle import oracle as O
+    tb = tok = 0
+    for pol, d in zip(POLICIES, DELTAS):
+        rec, _, _ = O.run(pol, B, d, kv, a, p, o, per_request=False)
+        tb += int(rec["T_busy"].sum())
+        tok += int(rec["token_adv"].sum())
+    return tb, tok
+
+
+def oracle_timed(a, p, o, B, kv, cores, pool):
+    chunks = [x for x in np.array_split(np.arange(len(a)), cores) if len(x)]
+    jobs = [(a[c], p[c], o[c], B, kv) for c in chunks]
+    t = time.perf_counter()
+    res = pool.map(_oracle_chunk, jobs)
+    dt = time.perf_counter() - t
+    return sum(r[0] for r in res), sum(r[1] for r in res), dt
+
+
+def cpu_model():
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu part")):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.processor() or platform.machine()
+
+
+# --------------------------------------------------------------- dist -------
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def reference_arm(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    wl = W.WORKLOADS[WID]
+    cores = os.cpu_count() or 1
+    per_core = 12
+    a, p, o = W.generate(WID, cores * per_core)
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(cores) as pool:
+        for _ in range(args.warmup):
+            oracle_timed(a, p, o, wl.B[0], wl.kv_caps[0], cores, pool)
+        tb_tot = tok_tot = 0
+        t_tot = 0.0
+        for _ in range(args.steps):
+            tb, tok, dt = oracle_timed(a, p, o, wl.B[0], wl.kv_caps[0], cores, pool)
+            tb_tot += tb
+            tok_tot += tok
+            t_tot += dt
+    value = tb_tot / t_tot
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t_tot / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
+        "data": "synthetic", "config": workload_config("cpu-oracle", wl, "n/a (CPU)"),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"first {cores * per_core} of {wl.n_instances} instances x 7 runs per step",
+                         "cpu": cpu_model()},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "token_advances_per_s": tok_tot / t_tot,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--kernel", choices=["step", "epoch"], default="step")
+    ap.add_argument("--instances", type=int, default=0, help="use only the first N instances (profiling)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return reference_arm(args)
+
+    world, rank, local = dist_env()
+    wl = W.WORKLOADS[WID]
+    n_inst = args.instances or wl.n_instances
+    B, kv = wl.B[0], wl.kv_caps[0]
+
+    # the oracle pool starts before the first CUDA call (spawned workers)
+    pool = None
+    cores = os.cpu_count() or 1
+    if rank == 0 and world >= 1 and not args.no_cpu_baseline:
+        pool = mp.get_context("spawn").Pool(cores)
+
+    import torch
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2608_02244_gb300 import sim
+
+    a_h, p_h, o_h = W.generate(WID, n_inst, replica=rank)
+    a = torch.from_numpy(a_h).cuda()
+    p = torch.from_numpy(p_h).cuda()
+    o = torch.from_numpy(o_h).cuda()
+    epoch = args.kernel == "epoch"
+    S = sim.Simulator(n_inst, wl.n_per_instance, B, wl.c, wl.tau, wl.p0, epoch=epoch, timing=True)
+    flush = torch.empty(64 * 2**20, dtype=torch.int32, device="cuda")   # 256 MiB > 129 MB L2
+    stream = torch.cuda.current_stream()
+
+    # warm-up (also yields the deterministic per-step unit counts)
+    for _ in range(max(args.warmup, 1)):
+        S.sweep_async(a, p, o, POLICIES, DELTAS, kv, per_request=True)
+    st, summ = sim.isjl_sim_metrics(S.handle)
+    if st != 0:
+        raise RuntimeError(f"device status {st}: {sim.isjl_status_string(st)}")
+    runs = [sim.summary_to_dict(summ[i]) for i in range(len(POLICIES))]
+    busy_per_step = sum(r["T_busy"] for r in runs)
+    tok_per_step = sum(r["token_adv"] for r in runs)
+    launches_per_step = sim.isjl_sim_last_launches(S.handle)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        uuid = None
+    sampler = ClockSampler(uuid)
+    time.sleep(0.4)
+    step_ms, sim_ms = [], []
+    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    t_wall = time.perf_counter()
+    for k in range(args.steps):
+        flush.zero_()                      # evict L2 between timed steps (outside the events)
+        ev0[k].record(stream)
+        S.sweep_async(a, p, o, POLICIES, DELTAS, kv, per_request=True)
+        ev1[k].record(stream)
+        kt = sim.isjl_sim_kernel_times(S.handle)   # waits for this step's events
+        sim_ms.append(kt[2])
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    wall = time.perf_counter() - t_wall
+    clocks = sampler.stop()
+    step_ms = [ev0[k].elapsed_time(ev1[k]) for k in range(args.steps)]
+    t_ms = sum(step_ms)
+
+    # e2e through the host-memory entry point: H2D of the inputs, sweep, D2H of the records
+    e2e = None
+    if not args.no_e2e:
+        pa, pp, po = (torch.from_numpy(x).pin_memory() for x in (a_h, p_h, o_h))
+        hrec = torch.empty(len(POLICIES) * n_inst * sim.RECORD_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
+        sim.isjl_sim_run_sweep_host(S.handle, POLICIES, DELTAS, kv, pa, pp, po, hrec)   # warm
+        torch.cuda.synchronize()
+        e2e_ms = []
+        for _ in range(args.steps):
+            t0 = time.perf_counter()
+            rc = sim.isjl_sim_run_sweep_host(S.handle, POLICIES, DELTAS, kv, pa, pp, po, hrec)
+            e2e_ms.append(1e3 * (time.perf_counter() - t0))
+            if rc != 0:
+                raise RuntimeError(f"host sweep status {rc}")
+        e2e = {"ms": sum(e2e_ms) / len(e2e_ms),
+               "h2d": 3 * a_h.nbytes, "d2h": hrec.numel()}
+
+    # max over ranks, sum of units
+    units = float(busy_per_step * args.steps)
+    if dist:
+        t = torch.tensor([t_ms, units, e2e["ms"] if e2e else 0.0], dtype=torch.float64, device="cuda")
+        tmax = t.clone()
+        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
+        tsum = t.clone()
+        dist.all_reduce(tsum, op=dist.ReduceOp.SUM)
+        t_ms_all, units_all, e2e_ms_all = float(tmax[0]), float(tsum[1]), float(tmax[2])
+    else:
+        t_ms_all, units_all, e2e_ms_all = t_ms, units, (e2e["ms"] if e2e else 0.0)
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        S.close()
+        return 0
+
+    value = units_all / (t_ms_all / 1e3)
+    sim_avg_ms = sum(sim_ms) / len(sim_ms)
+    sm_mhz = clocks.get("sm_mhz") or float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+                                            .get("clocks_under_load", {}).get("sm_mhz_median", 1417.0))
+    sms = torch.cuda.get_device_properties(local).multi_processor_count
+    peak_tops = sms * ALU_LANES_PER_SM * sm_mhz * 1e6 / 1e12
+    if epoch:
+        roofline = {"bound": "alu", "achieved": None, "peak": peak_tops, "unit": "Tops/s", "frac": None,
+                    "traffic": None, "kernel": "sim_kernel (epoch)",
+                    "note": "event-driven kernel: per-token work is replaced by closed forms; see the step kernel"}
+    else:
+        ops = OPS_PER_TOKEN_ADVANCE * tok_per_step + OPS_PER_BATCH_STEP * busy_per_step
+        achieved = ops / (sim_avg_ms / 1e3) / 1e12
+        roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s",
+                    "frac": achieved / peak_tops, "traffic": SIM_DRAM_BYTES_PER_LAUNCH,
+                    "kernel": "sim_kernel (step)", "ops_per_launch": ops,
+                    "peak_basis": f"{sms} SMs x {ALU_LANES_PER_SM} int32 lanes x {sm_mhz:.0f} MHz (median SM clock "
+                                  "sampled during the timed steps)",
+                    "sim_ms_per_launch": sim_avg_ms}
+
+    cpu = None
+    if pool is not None:
+        per_core = 8
+        sample_n = min(n_inst, cores * per_core)
+        tb, tok, dt = oracle_timed(a_h[:sample_n], p_h[:sample_n], o_h[:sample_n], B, kv, cores, pool)
+        pool.close()
+        cpu = {"value": tb / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"first {sample_n} of {n_inst} instances x {len(POLICIES)} runs ({dt:.1f} s wall)",
+               "cpu": cpu_model()}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t_ms_all / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+        "config": workload_config(args.kernel, W.WORKLOADS[WID] if n_inst == wl.n_instances else
+                                  W.Workload(3, "subset", n_inst, wl.n_per_instance, wl.seed, wl.B, wl.kv_caps,
+                                             wl.deltas), "flushed between steps (256 MiB write, outside the events)"),
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": ({"value": units_all / (e2e_ms_all / 1e3) / args.steps, "unit": UNIT,
+                 "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"]} if e2e else None),
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": {"sm_mhz": clocks.get("sm_mhz"), "sm_max_mhz": clocks.get("sm_max_mhz"),
+                   "reasons": clocks.get("reasons")},
+        "instances_per_s": world * n_inst * len(POLICIES) * args.steps / (t_ms_all / 1e3),
+        "token_advances_per_s": tok_per_step * world * args.steps / (t_ms_all / 1e3),
+        "kernel_ms": {"sim": sim_avg_ms},
+        "wall_s": wall,
+    }
+    print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+    S.close()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

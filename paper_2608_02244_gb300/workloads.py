@@ -89,8 +89,9 @@ def _lognormal_int(rng, shape, median, sigma, lo, hi):
     return np.clip(x, lo, hi).astype(np.int32)
 
 
-def _draw_chunk(wl: Workload, chunk: int, rows: int):
-    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([wl.seed, chunk])))
+def _draw_chunk(wl: Workload, chunk: int, rows: int, replica: int = 0):
+    key = [wl.seed, chunk] + ([replica] if replica else [])
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence(key)))
     n = wl.n_per_instance
     shape = (rows, n)
     if wl.wid == 1:
@@ -122,12 +123,13 @@ def _draw_chunk(wl: Workload, chunk: int, rows: int):
     return arrival, prompt, output
 
 
-def generate(wid: int, instances=None):
+def generate(wid: int, instances=None, replica: int = 0):
     """Return (arrival, prompt, output), each int32 of shape (len(instances), n).
 
     ``instances`` is None (all instances), an int m (the first m) or an
     iterable of instance ids.  Instance i is identical whichever way it is
-    requested.
+    requested.  ``replica`` r > 0 draws an independent set of the same shape
+    (seed sequence [seed, chunk, r]); multi-GPU runs give rank r replica r.
     """
     wl = WORKLOADS[wid]
     if instances is None:
@@ -147,7 +149,7 @@ def generate(wid: int, instances=None):
         # always draw the whole chunk: later arrays depend on how many values
         # the earlier draws consumed
         rows = min(per, wl.n_instances - int(c) * per)
-        arrs = _draw_chunk(wl, int(c), rows)
+        arrs = _draw_chunk(wl, int(c), rows, replica)
         for k in range(3):
             out[k][sel] = arrs[k][ids[sel] % per]
     return tuple(out)

@@ -1,0 +1,264 @@
+"""GPU (C ABI, CUDA kernels) against the CPU oracle, record by record.
+
+Integers (every counter and every per-request start / completion step) must
+be bit-exact; the fp64 cost fields within 1e-12 relative (they are computed
+from identical integers in the same order, so in practice they agree
+exactly).  Both kernel variants (per-step and event-driven) are checked.
+"""
+import numpy as np
+import pytest
+
+from conftest import cuda_available
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not cuda_available(), reason="needs a CUDA GPU")]
+
+INF = 2**31 - 1
+RTOL = 1e-12
+F64 = ("c_T", "tau_Q", "tau_E", "cost", "revenue", "profit", "throughput", "ael")
+
+
+@pytest.fixture(scope="module")
+def S():
+    from paper_2608_02244_gb300 import sim
+    sim.lib()
+    return sim
+
+
+@pytest.fixture(scope="module")
+def O(oracle_mod):
+    return oracle_mod
+
+
+def assert_records_equal(g, r, ctx=""):
+    """g: GPU records, r: oracle records (same shape, structured)."""
+    for f in r.dtype.names:
+        if f in F64:
+            np.testing.assert_allclose(g[f], r[f], rtol=RTOL, atol=0, err_msg=f"{ctx} {f}")
+        else:
+            np.testing.assert_array_equal(g[f], r[f], err_msg=f"{ctx} {f}")
+
+
+def run_both(S, O, a, p, o, B, policies, deltas, kv, epoch, per_request=True, max_steps=0, check=True):
+    n_inst, n = a.shape
+    sm = S.Simulator(n_inst, n, B, max_steps=max_steps, epoch=epoch)
+    try:
+        res = sm.sweep(a, p, o, policies, deltas, kv, per_request=per_request)
+    finally:
+        sm.close()
+    assert res["launches"] == 4
+    if check:
+        for i, (pol, d) in enumerate(zip(policies, deltas)):
+            rec, st, co = O.run(pol, B, d, kv, a, p, o, max_steps=max_steps, per_request=per_request)
+            assert_records_equal(res["records"][i], rec, f"{pol} d={d} epoch={epoch}")
+            if per_request:
+                np.testing.assert_array_equal(res["start"][i], st, err_msg=f"start {pol} {d}")
+                np.testing.assert_array_equal(res["completion"][i], co, err_msg=f"completion {pol} {d}")
+    return res
+
+
+EPOCHS = [False, True]
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_single_instance_workload(S, O, epoch):
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o = W.generate(1)
+    run_both(S, O, a, p, o, 32, ["fcfs", "ljf", "isjl", "isjl", "isjl"], [32, 32, 32, 0, INF], 2048, epoch)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+@pytest.mark.parametrize("B", [2, 3])
+@pytest.mark.parametrize("kv", [16, INF])
+def test_tiny_exhaustive_workload(S, O, epoch, B, kv):
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o = W.generate(2)
+    pols = ["isjl"] * 5 + ["fcfs", "ljf"]
+    ds = [0, 1, 2, 4, INF, 0, 0]
+    run_both(S, O, a, p, o, B, pols, ds, kv, epoch)
+
+
+def test_tiny_exhaustive_competitive_ratio_on_gpu(S, O):
+    """GPU makespans against the exhaustive optimum: B=2 meets 3/4 and CR(gamma)
+    everywhere; B=3 misses exactly on the recorded instances."""
+    import os
+    import sys
+    sys.path.insert(0, os.path.join(os.path.dirname(__file__), "golden"))
+    import make_cr_findings as F
+    from test_competitive_ratio import load_findings
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, out = W.generate(2)
+    o = p + out
+    rec = load_findings()
+    for B in (2, 3):
+        sm = S.Simulator(len(a), 6, B, epoch=True)
+        try:
+            res = sm.sweep(a, p, out, ["isjl"] * 5, list(F.DELTAS), INF)
+        finally:
+            sm.close()
+        for r, d in enumerate(F.DELTAS):
+            T = res["records"][r]["T_make"]
+            f34, fg = [], []
+            for i in range(len(o)):
+                topt = O.opt_makespan(a[i], o[i], B, d)
+                m34, mg = F.misses(topt, int(T[i]), int(o[i].max()), d)
+                if m34:
+                    f34.append(i)
+                if mg:
+                    fg.append(i)
+            if B == 2:
+                assert f34 == [] and fg == []
+            else:
+                assert f34 == rec[(3, d, "3/4")] and fg == rec[(3, d, "gamma")]
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_online_sweep_workload_subset(S, O, epoch):
+    """16 full-size instances (n = 1000, ragged against 32) of the online sweep."""
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o = W.generate(3, 16)
+    pols = ["fcfs", "ljf"] + ["isjl"] * 5
+    ds = [0, 0, 16, 64, 256, 1024, INF]
+    run_both(S, O, a, p, o, 256, pols, ds, 200_000, epoch)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_heavy_tail_workload_subset(S, O, epoch):
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o = W.generate(4, 48)
+    pols = ["fcfs", "ljf", "isjl", "isjl", "isjl"]
+    ds = [0, 0, 32, 128, 512]
+    run_both(S, O, a, p, o, 128, pols, ds, 65_536, epoch)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_large_instance_sample(S, O, epoch):
+    """One instance of n = 100,000 (radix-sort path, two-level pending set)."""
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o = W.generate(5, [7])
+    run_both(S, O, a, p, o, 512, ["fcfs", "ljf", "isjl"], [256, 256, 256], 1_000_000, epoch)
+
+
+def test_online_sweep_full_size_sampled(S, O):
+    """The benchmark's launch: all 10,000 instances x 7 runs in one sweep;
+    sampled instances against the oracle, invariants on every record."""
+    from paper_2608_02244_gb300 import workloads as W
+    wl = W.WORKLOADS[3]
+    a, p, o = W.generate(3)
+    pols = ["fcfs", "ljf"] + ["isjl"] * 5
+    ds = [0, 0, 16, 64, 256, 1024, INF]
+    for epoch in EPOCHS:
+        sm = S.Simulator(wl.n_instances, wl.n_per_instance, 256, epoch=epoch)
+        try:
+            res = sm.sweep(a, p, o, pols, ds, 200_000, per_request=True)
+        finally:
+            sm.close()
+        assert res["status"] == 0
+        R = res["records"]
+        assert (R["status"] == 0).all()
+        assert (R["W"] == R["Q"] + R["E"]).all() and (R["token_adv"] == R["O"]).all()
+        assert (R["violations"][1:] == 0).all() and (R["kv_violations"] == 0).all()
+        assert (R["peak_kv"] <= 200_000).all() and (R["peak_batch"] <= 256).all()
+        sample = [0, 1, 977, 2048, 4099, 5555, 8191, 9999]
+        for i, (pol, d) in enumerate(zip(pols, ds)):
+            rec, st, co = O.run(pol, 256, d, 200_000, a[sample], p[sample], o[sample])
+            assert_records_equal(R[i][sample], rec, f"full {pol} {d} epoch={epoch}")
+            np.testing.assert_array_equal(res["start"][i][sample], st)
+            np.testing.assert_array_equal(res["completion"][i][sample], co)
+            # summaries: exact integer totals, fp64 within tolerance
+            s = res["summaries"][i]
+            assert s["T_busy"] == int(R[i]["T_busy"].sum()) and s["E"] == int(R[i]["E"].sum())
+            assert s["n_ok"] == wl.n_instances and s["status"] == 0
+            np.testing.assert_allclose(s["cost"], R[i]["cost"].sum(), rtol=1e-12)
+
+
+# ---- edge cases -------------------------------------------------------------
+def _inst(rows):
+    a = np.array([r[0] for r in rows], np.int32)
+    p = np.array([r[1] for r in rows], np.int32)
+    o = np.array([r[2] for r in rows], np.int32)
+    return a, p, o
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_edge_shapes(S, O, epoch):
+    rng = np.random.default_rng(7)
+    cases = []
+    # n = 1; B = 1; n = 33 (two bitset words); B = 512 with few requests; idle gaps
+    for n, B in [(1, 1), (1, 4), (33, 1), (33, 3), (64, 512), (200, 64), (97, 2)]:
+        a = np.sort(rng.integers(0, 400, (5, n)), axis=1).astype(np.int32)
+        p = rng.integers(0, 30, (5, n)).astype(np.int32)
+        o = rng.integers(1, 90, (5, n)).astype(np.int32)
+        cases.append((a, p, o, B))
+    for a, p, o, B in cases:
+        kv = int((p + o).max()) + 50
+        run_both(S, O, a, p, o, B, ["fcfs", "ljf", "isjl", "isjl", "isjl"], [0, 0, 0, 5, INF], kv, epoch)
+        run_both(S, O, a, p, o, B, ["isjl", "isjl"], [3, 40], INF, epoch)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_radix_path_small_count(S, O, epoch):
+    """n = 4097 takes the radix sort; long idle gaps between arrivals."""
+    rng = np.random.default_rng(8)
+    n = 4097
+    a = np.sort(rng.integers(0, 30000, (2, n)), axis=1).astype(np.int32)
+    p = rng.integers(0, 200, (2, n)).astype(np.int32)
+    o = rng.integers(1, 300, (2, n)).astype(np.int32)
+    run_both(S, O, a, p, o, 40, ["fcfs", "ljf", "isjl", "isjl"], [0, 0, 60, INF], 3000, epoch)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_error_statuses(S, O, epoch):
+    a = np.zeros((4, 3), np.int32)
+    p = np.zeros((4, 3), np.int32)
+    o = np.array([[3, 2, 1], [3, 0, 1], [3, 2, 1], [9, 2, 1]], np.int32)
+    a[2] = [0, 2, 1]               # decreasing arrivals
+    res = run_both(S, O, a, p, o, 2, ["fcfs", "isjl"], [0, 1], 8, epoch, check=False)
+    R = res["records"]
+    assert list(R["status"][0]) == [0, 2, 1, 2]   # ok, o=0 infeasible, invalid, o > kv infeasible
+    assert res["status"] in (1, 2)
+    for i, (pol, d) in enumerate([("fcfs", 0), ("isjl", 1)]):
+        rec, _, _ = O.run(pol, 2, d, 8, a, p, o)
+        np.testing.assert_array_equal(R[i]["status"], rec["status"])
+        assert_records_equal(R[i][:1], rec[:1])
+    # the step guard returns an error status instead of trapping
+    res = run_both(S, O, a[:1], p[:1], o[:1], 2, ["isjl"], [0], 8, epoch, max_steps=2, check=False)
+    assert res["records"][0]["status"][0] == 5 and res["status"] == 5
+
+
+def test_invalid_arguments_rejected(S):
+    import torch
+    sm = S.Simulator(1, 4, 2)
+    try:
+        x = torch.zeros(4, dtype=torch.int32, device="cuda")
+        rec, _, _ = sm.buffers(1, False)
+        assert S.isjl_sim_run(sm.handle, 2, -1, 10, x, x, x, rec) == S.ISJL_ERR_INVALID_ARG
+        assert S.isjl_sim_run(sm.handle, 2, 1, 0, x, x, x, rec) == S.ISJL_ERR_INVALID_ARG
+        assert S.isjl_sim_run(sm.handle, 7, 1, 10, x, x, x, rec) == S.ISJL_ERR_INVALID_ARG
+    finally:
+        sm.close()
+    with pytest.raises(S.IsjlError):
+        S.isjl_sim_create(1, 4, 513)
+    with pytest.raises(S.IsjlError):
+        S.isjl_sim_create(0, 4, 2)
+
+
+def test_sweep_equals_single_runs_and_host_entry_point(S):
+    import torch
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o = W.generate(3, 8)
+    pols, ds = ["fcfs", "isjl", "isjl"], [0, 64, INF]
+    sm = S.Simulator(8, 1000, 256, epoch=True)
+    try:
+        res = sm.sweep(a, p, o, pols, ds, 200_000)
+        for i, (pol, d) in enumerate(zip(pols, ds)):
+            one = sm.sweep(a, p, o, [pol], [d], 200_000)
+            assert res["records"][i].tobytes() == one["records"][0].tobytes()
+        pin = [torch.from_numpy(np.ascontiguousarray(x)).pin_memory() for x in (a, p, o)]
+        hrec = torch.empty(len(pols) * 8 * S.RECORD_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
+        st = S.isjl_sim_run_sweep_host(sm.handle, pols, ds, 200_000, *pin, hrec)
+        assert st == 0
+        host = hrec.numpy().view(S.RECORD_DTYPE).reshape(len(pols), 8)
+        assert host.tobytes() == res["records"].tobytes()
+    finally:
+        sm.close()
