@@ -10,13 +10,19 @@
 //   cost      W += |S| max r, E += sum (max r - r_i), extent, T_busy
 //             (Section 5, Eq. batch-cost-progress and the decomposition)
 //
-// Layout: worker (batch slot) w lives in lane w / SPL, register slot w % SPL,
-// so a warp covers B <= 32 * SPL workers; the max / min / sum of the step are
-// warp reductions (REDUX).  The pending queue is a bitset over the request
-// positions of the instance sorted by (o desc, index asc): the longest pending
-// request is the lowest set bit (two levels: 32-bit words plus a summary word
-// per 32 words, in shared memory).  ISJL plans are per-worker FIFO lists
-// linked through a global scratch array.
+// Layout.  Worker (batch slot) w lives in lane w % 32, register row w / 32,
+// so a warp holds B <= 32 * SPL workers.  The step kernel advances every
+// slot each step, straight-line: an idle slot carries the sentinel progress
+// IDLE + k, which is below every real progress as a signed value, above it as
+// an unsigned value, and known, so the step's max (signed), min (unsigned) and
+// sum (corrected by the idle count) need no per-slot predicate.  Values that
+// change only at events (next arrival, earliest completion, start range, KV
+// reservation) are kept as warp-uniform scalars, so a step without an event
+// runs no warp reduction beyond the three of the step cost.  The pending
+// queue is a bitset over the instance's request positions sorted by
+// (o desc, index asc) -- the longest pending request is the lowest set bit --
+// with a summary word per 32 words, in shared memory.  ISJL plans are
+// per-worker FIFO lists linked through a global scratch array.
 //
 // Two variants share the admission code:
 //   step kernel   advances every running request each step (the literal loop)
@@ -36,37 +42,33 @@ namespace isjl {
 namespace {
 
 constexpr int32_t kNone = -1;
+constexpr int32_t kIdle = -(1 << 30);   // idle-slot progress sentinel base
 
 struct WarpSmem {
     int32_t *sjob;    // [B] request running on worker w
     int32_t *shead;   // [B] next ISJL plan entry of worker w (kNone = none)
     int32_t *stail;   // [B] last plan entry of worker w
     int32_t *slong;   // [B] long request o_j planned on worker j (1 <= j < n_long)
+    int32_t *srem;    // [B] ISJL packing budget left on worker w (Phase ONE only)
+    int32_t *spsum;   // [B] ISJL pack sum on worker w (Phase ONE only)
     uint32_t *pend0;  // [words0] bit p: sorted position p is pending
     uint32_t *pend1;  // [words1] bit w: pend0[w] != 0
 };
 
 __host__ __device__ inline int smem_words_per_warp(int B, int words0, int words1) {
-    int w = 4 * B + words0 + words1;
+    int w = 6 * B + words0 + words1;
     return (w + 3) & ~3;  // keep every warp's block 16-byte aligned
 }
 
-template <int SPL>
-__device__ __forceinline__ int lowest_worker(uint32_t m) {
-    const unsigned b = __ballot_sync(kFull, m != 0u);
-    if (!b) return -1;
-    const int l = __ffs(b) - 1;
-    const uint32_t mm = __shfl_sync(kFull, m, l);
-    return l * SPL + (__ffs(mm) - 1);
+// lowest / highest worker whose row bit is set in the per-lane mask m
+__device__ __forceinline__ int lowest_worker(uint32_t m, int lane) {
+    const int v = m ? ((__ffs(m) - 1) << 5) + lane : INT_MAX;
+    const int r = __reduce_min_sync(kFull, v);
+    return r == INT_MAX ? -1 : r;
 }
-
-template <int SPL>
-__device__ __forceinline__ int highest_worker(uint32_t m) {
-    const unsigned b = __ballot_sync(kFull, m != 0u);
-    if (!b) return -1;
-    const int l = 31 - __clz(b);
-    const uint32_t mm = __shfl_sync(kFull, m, l);
-    return l * SPL + (31 - __clz(mm));
+__device__ __forceinline__ int highest_worker(uint32_t m, int lane) {
+    const int v = m ? ((31 - __clz(m)) << 5) + lane : -1;
+    return __reduce_max_sync(kFull, v);
 }
 
 __device__ __forceinline__ int64_t warp_sum64(int64_t v) {
@@ -147,7 +149,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     const int32_t *__restrict__ perm = A.perm + base;
     const int32_t *__restrict__ osrt = A.osorted + base;
     const int32_t *__restrict__ posof = A.posof + base;
-    int32_t *__restrict__ pnext = A.plan_next + gwarp * (int64_t)n;
+    int32_t *pnext = A.plan_next + gwarp * (int64_t)n;
     const int64_t out_off = (int64_t)run * A.n_inst * n + base;
     int32_t *st_out = A.start_out ? A.start_out + out_off : nullptr;
     int32_t *co_out = A.compl_out ? A.compl_out + out_off : nullptr;
@@ -156,11 +158,12 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 
     int64_t status = is.status;
     if (status == ISJL_OK && (int64_t)is.maxo > kv_cap) status = ISJL_ERR_INFEASIBLE;
-    // step counters are int32: every schedule ends by sum o + max arrival
-    if (status == ISJL_OK && is.O + (int64_t)is.maxA + 1 > (int64_t)INT_MAX) status = ISJL_ERR_INVALID_ARG;
+    // every schedule ends by sum o + max arrival; the idle sentinel needs steps < 2^30
+    if (status == ISJL_OK && is.O + (int64_t)is.maxA + 1 >= (int64_t)(1 << 30)) status = ISJL_ERR_INVALID_ARG;
 
-    int64_t W = 0, E = 0, Tb = 0, tok = 0, sumc = 0, sumext = 0, maxext = 0, viol = 0, kvviol = 0;
-    int64_t peakkv = 0, peakb = 0, Tmake = 0;
+    // W = sum |S| max r; R = sum over steps of sum r (E = W - R at the end)
+    int64_t W = 0, R = 0, E = 0, sumc = 0, sumext = 0, peakkv = 0;
+    int32_t Tb = 0, tok = 0, maxext = 0, viol = 0, peakb = 0, Tmake = 0, kvviol = 0;
 
     if (status == ISJL_OK) {
         for (int w = lane; w < words0; w += 32) S.pend0[w] = 0u;
@@ -168,76 +171,111 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         for (int w = lane; w < B; w += 32) { S.shead[w] = kNone; S.stail[w] = kNone; S.slong[w] = kNone; }
         __syncwarp();
 
-        // per-lane worker slots: a_ = progress (step kernel) or start step (epoch kernel)
-        int32_t a_[SPL], oo[SPL];
+        // worker w = r * 32 + lane: sa = progress (step kernel) or start step
+        // (epoch kernel), sc = completion step (INT_MAX when idle)
+        int32_t sa[SPL], sc[SPL];
 #pragma unroll
-        for (int r = 0; r < SPL; ++r) { a_[r] = 0; oo[r] = 0; }
+        for (int r = 0; r < SPL; ++r) { sa[r] = kIdle; sc[r] = INT_MAX; }
         uint32_t busy = 0u, resv = 0u;
-        const int nv = B - lane * SPL;
-        const uint32_t vmask = nv <= 0 ? 0u : (nv >= SPL ? (SPL == 32 ? ~0u : ((1u << SPL) - 1u)) : ((1u << nv) - 1u));
+        int32_t lane_cmin = INT_MAX;                 // earliest completion among this lane's workers
+        int32_t lane_smin = INT_MAX, lane_smax = INT_MIN;   // start range (epoch kernel)
+        const int nrow = (B - lane + 31) >> 5;       // rows holding a valid worker for this lane
+        const uint32_t vmask = nrow >= 32 ? ~0u : ((1u << nrow) - 1u);
+        const int32_t alpha32 = (int32_t)min(alpha, (int64_t)INT_MAX);
 
         int32_t k = 0, rel = 0, fcfs = 0, done = 0, run_cnt = 0, pend = 0;
         int64_t kv_sum = 0, sum_st = 0;
+        // uniform caches, changed only at events
+        int32_t next_arr = n > 0 ? arr[0] : INT_MAX;   // arrival of the next unreleased request
+        int32_t cmin = INT_MAX;                        // earliest completion step of the running set
+        int32_t smin = INT_MAX, smax = INT_MIN;        // start range of the running set (epoch kernel)
+        int32_t kv_over = 0;                           // reserved KV above the cap (never, by construction)
         int32_t plan_left = 0, t0 = 0, d1 = 0, L1 = kNone, nlong = 0;
-        bool L1_started = true, adm_blocked = false;
+        bool L1_started = true;
         bool broken = false;   // an internal invariant failed: stop without touching memory
         const int64_t max_steps = A.max_steps > 0 ? A.max_steps : (is.O + (int64_t)is.maxA + 1);
+        const int32_t step_guard = (int32_t)min(max_steps + 1, (int64_t)INT_MAX);
 
+        auto recompute_lane = [&]() {
+            lane_cmin = INT_MAX;
+            if (EPOCH) { lane_smin = INT_MAX; lane_smax = INT_MIN; }
+#pragma unroll
+            for (int r = 0; r < SPL; ++r) {
+                if (busy >> r & 1u) {
+                    lane_cmin = min(lane_cmin, sc[r]);
+                    if (EPOCH) { lane_smin = min(lane_smin, sa[r]); lane_smax = max(lane_smax, sa[r]); }
+                }
+            }
+        };
         // start request e (length oe) on worker w at step k
         auto start = [&](int e, int oe, int w) {
             run_cnt++;
             kv_sum += oe;
-            if (EPOCH) sum_st += k;
-            const int l = w / SPL, rr = w - l * SPL;
-            if (lane == l) {
+            cmin = min(cmin, k + oe);
+            peakkv = max(peakkv, kv_sum);
+            peakb = max(peakb, run_cnt);
+            kv_over = kv_sum > kv_cap;
+            if (EPOCH) { sum_st += k; smin = min(smin, k); smax = k; }
+            const int owner = w & 31, row = w >> 5;
+            if (lane == owner) {
 #pragma unroll
                 for (int r = 0; r < SPL; ++r)
-                    if (r == rr) { a_[r] = EPOCH ? k : 0; oo[r] = oe; }
-                busy |= 1u << rr;
+                    if (r == row) { sa[r] = EPOCH ? k : 0; sc[r] = k + oe; }
+                busy |= 1u << row;
+                lane_cmin = min(lane_cmin, k + oe);
+                if (EPOCH) { lane_smin = min(lane_smin, k); lane_smax = max(lane_smax, k); }
                 S.sjob[w] = e;
                 if (st_out) st_out[e] = k;
             }
+            if (!EPOCH && run_cnt == 1) {
+                // first start after an empty batch: idle slots take the current sentinel
+#pragma unroll
+                for (int r = 0; r < SPL; ++r)
+                    if (!(busy >> r & 1u)) sa[r] = kIdle + k - 1;
+            }
         };
-        // requests of the workers in fin (per lane) complete at step c
-        auto retire = [&](uint32_t fin, int32_t c) {
-            if (!__ballot_sync(kFull, fin != 0u)) return;
+        // requests completing at step c leave their workers
+        auto retire = [&](int32_t c) {
+            uint32_t fm = 0u;
             int nf = 0, of = 0;
             int64_t sf = 0;
 #pragma unroll
             for (int r = 0; r < SPL; ++r) {
-                if (fin >> r & 1u) {
+                if ((busy >> r & 1u) && sc[r] == c) {
+                    fm |= 1u << r;
                     nf++;
-                    of += oo[r];
-                    if (EPOCH) sf += a_[r];
-                    if (co_out) co_out[S.sjob[lane * SPL + r]] = c;
+                    of += EPOCH ? sc[r] - sa[r] : sa[r];
+                    if (EPOCH) sf += sa[r];
+                    if (co_out) co_out[S.sjob[(r << 5) + lane]] = c;
+                    sc[r] = INT_MAX;
+                    if (!EPOCH) sa[r] = kIdle + c - 1;   // sentinel of the step just served
                 }
             }
-            busy &= ~fin;
+            busy &= ~fm;
+            if (fm) recompute_lane();
             nf = (int)__reduce_add_sync(kFull, (unsigned)nf);
             of = (int)__reduce_add_sync(kFull, (unsigned)of);
             if (EPOCH) sum_st -= warp_sum64(sf);
             done += nf;
             run_cnt -= nf;
             kv_sum -= of;
+            kv_over = kv_sum > kv_cap;
             sumc += (int64_t)nf * c;
             Tmake = c;
-            adm_blocked = false;
+            cmin = __reduce_min_sync(kFull, lane_cmin);
+            if (EPOCH) {
+                smin = __reduce_min_sync(kFull, lane_smin);
+                smax = __reduce_max_sync(kFull, lane_smax);
+            }
         };
         // A_max(k): largest progress among running requests (0 if none)
         auto amax_now = [&]() -> int64_t {
             if (run_cnt == 0) return 0;
-            if (EPOCH) {
-                int m = INT_MAX;
+            if (EPOCH) return (int64_t)k - smin;
+            int m = 0;
 #pragma unroll
-                for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = min(m, a_[r]);
-                m = __reduce_min_sync(kFull, m);
-                return (int64_t)k - m;
-            } else {
-                int m = 0;
-#pragma unroll
-                for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = max(m, a_[r]);
-                return (int64_t)__reduce_max_sync(kFull, m);
-            }
+            for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = max(m, sa[r]);
+            return (int64_t)__reduce_max_sync(kFull, m);
         };
 
         // ISJL Phase ONE at a stage start (Algorithm 2 with beta = alpha)
@@ -253,13 +291,12 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             // M = min{B, #{o > alpha}} over Q(k)
             const int cnt_long = bs_count_below(S, words0, first_pos_le(osrt, n, alpha), lane);
             const int nl = min(B, cnt_long);
-            int32_t rem[SPL], psum[SPL];   // packing budget left / pack sum per worker
-#pragma unroll
-            for (int r = 0; r < SPL; ++r) {
-                const int w = lane * SPL + r;
-                rem[r] = (w >= nl && w < B) ? (int32_t)alpha : -1;   // workers M+1..B: alpha
-                psum[r] = 0;
+            // packing budget left / pack sum per worker, in shared memory
+            for (int w = lane; w < B; w += 32) {
+                S.srem[w] = w >= nl ? (int32_t)alpha : -1;   // workers M+1..B: alpha
+                S.spsum[w] = 0;
             }
+            __syncwarp();
             // the long requests o_1..o_M leave Q; worker j's budget cap_j
             int p = -1;
             int64_t o_last = o1;
@@ -275,11 +312,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 } else {
                     const int64_t cap = min(2 * alpha, o1 - oe + alpha);
                     if (lane == 0) S.slong[j] = e;
-                    const int l = j / SPL, rr = j - l * SPL;
-                    if (lane == l) {
-#pragma unroll
-                        for (int r = 0; r < SPL; ++r) if (r == rr) rem[r] = (int32_t)cap;
-                    }
+                    if (lane == 0) S.srem[j] = (int32_t)cap;
                 }
                 o_last = oe;
             }
@@ -288,8 +321,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             const int64_t theta = min(2 * alpha, o1 - o_last + alpha);
             // first fit of the shorter requests, in sorted order
             int maxrem = -1;
-#pragma unroll
-            for (int r = 0; r < SPL; ++r) maxrem = max(maxrem, rem[r]);
+            for (int w = lane; w < B; w += 32) maxrem = max(maxrem, S.srem[w]);
             maxrem = __reduce_max_sync(kFull, maxrem);
             int q = -1;
             for (;;) {
@@ -303,13 +335,13 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 uint32_t mA = 0u, mB = 0u;
 #pragma unroll
                 for (int r = 0; r < SPL; ++r) {
-                    const int w = lane * SPL + r;
-                    const bool fits = rem[r] >= oe;
+                    const int w = (r << 5) + lane;
+                    const bool fits = w < B && S.srem[w] >= oe;
                     if (fits && w >= nl && w < B) mA |= 1u << r;
                     if (fits && w >= 1 && w < nl) mB |= 1u << r;
                 }
-                int w = lowest_worker<SPL>(mA);                 // workers M+1..B first
-                if (w < 0) w = highest_worker<SPL>(mB);         // then M, M-1, ..., 2
+                int w = lowest_worker(mA, lane);                // workers M+1..B first
+                if (w < 0) w = highest_worker(mB, lane);        // then M, M-1, ..., 2
                 if (w < 0) { broken = true; return; }
                 if (lane == 0) {
                     const int tl = S.stail[w];
@@ -317,17 +349,12 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     S.stail[w] = e;
                     pnext[e] = kNone;
                 }
-                const int l = w / SPL, rr = w - l * SPL;
-                if (lane == l) {
-#pragma unroll
-                    for (int r = 0; r < SPL; ++r) if (r == rr) { rem[r] -= oe; psum[r] += oe; }
-                }
+                if (lane == 0) { S.srem[w] -= oe; S.spsum[w] += oe; }
                 bs_clear(S, q, lane);   // includes __syncwarp
                 pend--;
                 plan_left++;
                 maxrem = -1;
-#pragma unroll
-                for (int r = 0; r < SPL; ++r) maxrem = max(maxrem, rem[r]);
+                for (int w2 = lane; w2 < B; w2 += 32) maxrem = max(maxrem, S.srem[w2]);
                 maxrem = __reduce_max_sync(kFull, maxrem);
             }
             // worker j (2..M) runs o_j after its pack
@@ -342,17 +369,13 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             plan_left += nl;
             // o_1 waits d1 = min{max{max_j sum(w_j) - alpha, 0}, alpha}, j = 2..M
             int mx = 0;
-#pragma unroll
-            for (int r = 0; r < SPL; ++r) {
-                const int w = lane * SPL + r;
-                if (w >= 1 && w < nl) mx = max(mx, psum[r]);
-            }
+            for (int w = 1 + lane; w < nl; w += 32) mx = max(mx, S.spsum[w]);
             mx = __reduce_max_sync(kFull, mx);
             d1 = (int32_t)min(max((int64_t)mx - alpha, (int64_t)0), alpha);
             resv = 0u;
 #pragma unroll
             for (int r = 0; r < SPL; ++r) {
-                const int w = lane * SPL + r;
+                const int w = (r << 5) + lane;
                 if (w < B && S.shead[w] >= 0) resv |= 1u << r;
             }
             L1_started = false;
@@ -365,7 +388,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 while (run_cnt < B && fcfs < rel) {
                     const int oe = oarr[fcfs];
                     if (kv_sum + oe > kv_cap) break;
-                    const int w = lowest_worker<SPL>(vmask & ~busy);
+                    const int w = lowest_worker(vmask & ~busy, lane);
                     if (w < 0) { broken = true; return; }
                     start(fcfs, oe, w);
                     fcfs++;
@@ -380,7 +403,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     const int oe = osrt[p];
                     if (kv_sum + oe > kv_cap) break;
                     const int e = perm[p];
-                    const int w = lowest_worker<SPL>(vmask & ~busy);
+                    const int w = lowest_worker(vmask & ~busy, lane);
                     if (w < 0) { broken = true; return; }
                     bs_clear(S, p, lane);
                     pend--;
@@ -395,13 +418,9 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     // plan starts, workers in order
                     uint32_t cand = resv & ~busy;
                     for (;;) {
-                        const unsigned b = __ballot_sync(kFull, cand != 0u);
-                        if (!b) break;
-                        const int l = __ffs(b) - 1;
-                        const uint32_t m = __shfl_sync(kFull, cand, l);
-                        const int rr = __ffs(m) - 1;
-                        const int w = l * SPL + rr;
-                        if (lane == l) cand &= ~(1u << rr);
+                        const int w = lowest_worker(cand, lane);
+                        if (w < 0) break;
+                        if (lane == (w & 31)) cand &= ~(1u << (w >> 5));
                         const int e = S.shead[w];
                         if (w == 0 && e == L1) {
                             const bool over = ((int64_t)k >= (int64_t)t0 + d1) || (k > t0 && nothing_runs);
@@ -414,7 +433,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         __syncwarp();
                         if (lane == 0) { S.shead[w] = nx; if (nx < 0) S.stail[w] = kNone; }
                         __syncwarp();
-                        if (nx < 0 && lane == l) resv &= ~(1u << rr);
+                        if (nx < 0 && lane == (w & 31)) resv &= ~(1u << (w >> 5));
                         plan_left--;
                         if (e == L1) L1_started = true;
                         start(e, oe, w);
@@ -424,7 +443,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     // Phase TWO: longest released request onto a free worker
                     int p = -1;
                     while (pend > 0) {
-                        const int w = lowest_worker<SPL>(vmask & ~busy & ~resv);
+                        const int w = lowest_worker(vmask & ~busy & ~resv, lane);
                         if (w < 0) break;
                         p = bs_next(S, words0, words1, p + 1, lane);
                         if (p >= n) { broken = true; return; }
@@ -439,116 +458,105 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             }
         };
 
-        for (;;) {
-            if ((int64_t)k > max_steps) { status = ISJL_ERR_STEP_LIMIT; break; }
-            // release: arrivals are non-decreasing, so the released requests are a prefix
-            if (rel < n && arr[rel] <= k) {
-                adm_blocked = false;
-                for (;;) {
-                    const int i = rel + lane;
-                    const bool ok = i < n && arr[i] <= k;
-                    const unsigned b = __ballot_sync(kFull, ok);
-                    if (ok && policy != ISJL_POLICY_FCFS) {
-                        const int p = posof[i];
-                        atomicOr(&S.pend0[p >> 5], 1u << (p & 31));
-                        atomicOr(&S.pend1[p >> 10], 1u << ((p >> 5) & 31));
-                    }
-                    const int c = __popc(b);
-                    rel += c;
-                    pend += c;
-                    if (c < 32) break;
+        // release every request with A_i <= k (a prefix: arrivals are non-decreasing)
+        auto release = [&]() {
+            for (;;) {
+                const int i = rel + lane;
+                const bool ok = i < n && arr[i] <= k;
+                const unsigned b = __ballot_sync(kFull, ok);
+                if (ok && policy != ISJL_POLICY_FCFS) {
+                    const int p = posof[i];
+                    atomicOr(&S.pend0[p >> 5], 1u << (p & 31));
+                    atomicOr(&S.pend1[p >> 10], 1u << ((p >> 5) & 31));
                 }
-                __syncwarp();
+                const int c = __popc(b);
+                rel += c;
+                pend += c;
+                if (c < 32) break;
             }
-            if (EPOCH) {
-                uint32_t fin = 0u;
-#pragma unroll
-                for (int r = 0; r < SPL; ++r)
-                    if ((busy >> r & 1u) && a_[r] + oo[r] == k) fin |= 1u << r;
-                retire(fin, k);
-            }
-            if (done == n) break;
-            if (!EPOCH && policy == ISJL_POLICY_ISJL && !L1_started && k == t0 + d1) adm_blocked = false;
-            if (EPOCH || !adm_blocked) {
-                admit();
-                adm_blocked = true;
-                if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
-            }
+            __syncwarp();
+            next_arr = rel < n ? arr[rel] : INT_MAX;
+        };
 
-            if (!EPOCH) {
+        if (!EPOCH) {
+            // ---------------------------------------------------- step kernel
+            int32_t next_check = 0;   // the next step needing release / admission / the guard
+            unsigned idle_slots = 0u; // idle slots inside the used rows
+            for (;;) {
+                if (k >= next_check) {
+                    if (k >= step_guard) { status = ISJL_ERR_STEP_LIMIT; break; }
+                    if (done == n) break;
+                    if (k >= next_arr) release();
+                    admit();
+                    if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
+                    next_check = next_arr;
+                    if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) next_check = min(next_check, t0 + d1);
+                    next_check = min(next_check, step_guard);
+                    idle_slots = (unsigned)(SPL * 32 - run_cnt);
+                }
                 if (run_cnt > 0) {
-                    // advance every running request by one token
-                    int rmax = 0, rmin = INT_MAX;
-                    unsigned rsum = 0u;
-                    uint32_t fin = 0u;
+                    // advance every running request by one token: r_i = a_i + 1
+                    // (all rows straight-line; idle slots advance their sentinel)
+                    int mx = INT_MIN;
+                    unsigned mn = 0xffffffffu, sm = 0u;
 #pragma unroll
                     for (int r = 0; r < SPL; ++r) {
-                        const bool bz = busy >> r & 1u;
-                        const int rr = a_[r] + 1;          // token index processed now
-                        if (bz) {
-                            a_[r] = rr;
-                            rmax = max(rmax, rr);
-                            rmin = min(rmin, rr);
-                            rsum += (unsigned)rr;
-                            if (rr == oo[r]) fin |= 1u << r;
-                        }
+                        const int a = sa[r] + 1;
+                        sa[r] = a;
+                        mx = max(mx, a);
+                        mn = min(mn, (unsigned)a);
+                        sm += (unsigned)a;
                     }
-                    rmax = __reduce_max_sync(kFull, rmax);
-                    rmin = __reduce_min_sync(kFull, rmin);
-                    rsum = __reduce_add_sync(kFull, rsum);
-                    const int64_t cnt = run_cnt;
-                    W += cnt * rmax;
-                    E += cnt * rmax - (int64_t)rsum;
-                    const int64_t ext = rmax - rmin;
+                    mx = __reduce_max_sync(kFull, mx);
+                    mn = __reduce_min_sync(kFull, mn);
+                    sm = __reduce_add_sync(kFull, sm);
+                    sm -= idle_slots * (unsigned)(kIdle + k);     // idle slots each added kIdle + k
+                    const int ext = mx - (int)mn;
+                    W += (int64_t)run_cnt * mx;                   // |S| max r
+                    R += (int64_t)(int32_t)sm;                    // sum r
                     sumext += ext;
                     maxext = max(maxext, ext);
-                    viol += ext > alpha;
-                    kvviol += kv_sum > kv_cap;
-                    peakkv = max(peakkv, kv_sum);
-                    peakb = max(peakb, cnt);
+                    viol += ext > alpha32;
                     Tb++;
-                    tok += cnt;
-                    retire(fin, k + 1);
-                }
-                k++;
-            } else {
-                // next event: arrival, completion or the end of o_1's delay
-                int64_t nxt = rel < n ? (int64_t)arr[rel] : INT64_MAX;
-                int mc = INT_MAX, mns = INT_MAX, mxs = INT_MIN;
-#pragma unroll
-                for (int r = 0; r < SPL; ++r) {
-                    if (busy >> r & 1u) {
-                        mc = min(mc, a_[r] + oo[r]);
-                        mns = min(mns, a_[r]);
-                        mxs = max(mxs, a_[r]);
+                    tok += run_cnt;
+                    kvviol += kv_over;
+                    if (k + 1 == cmin) {
+                        retire(k + 1);
+                        next_check = k + 1;
+                        idle_slots = (unsigned)(SPL * 32 - run_cnt);
                     }
                 }
-                mc = __reduce_min_sync(kFull, mc);
-                mns = __reduce_min_sync(kFull, mns);
-                mxs = __reduce_max_sync(kFull, mxs);
-                if (run_cnt > 0) nxt = min(nxt, (int64_t)mc);
-                if (policy == ISJL_POLICY_ISJL && !L1_started && (int64_t)t0 + d1 > k)
-                    nxt = min(nxt, (int64_t)t0 + d1);
-                if (nxt == INT64_MAX) { status = ISJL_ERR_STEP_LIMIT; break; }   // cannot progress
+                k++;
+            }
+            E = W - R;
+        } else {
+            // --------------------------------------------------- epoch kernel
+            for (;;) {
+                if ((int64_t)k > max_steps) { status = ISJL_ERR_STEP_LIMIT; break; }
+                if (k >= next_arr) release();
+                if (k == cmin) retire(k);
+                if (done == n) break;
+                admit();
+                if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
+                // next event: arrival, completion or the end of o_1's delay
+                int32_t nxt = min(next_arr, cmin);
+                if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) nxt = min(nxt, t0 + d1);
+                if (nxt == INT_MAX) { status = ISJL_ERR_STEP_LIMIT; break; }   // cannot progress
                 if (run_cnt > 0) {
                     const int64_t L = nxt - k, s = run_cnt;
-                    const int64_t m0 = (int64_t)k - mns + 1;       // max r at step k
-                    const int64_t n0 = (int64_t)k - mxs + 1;       // min r at step k
+                    const int64_t m0 = (int64_t)k - smin + 1;       // max r at step k
+                    const int32_t ext = smax - smin;                // max r - min r
                     const int64_t sr = s * ((int64_t)k + 1) - sum_st;   // sum r at step k
                     W += s * (L * m0 + L * (L - 1) / 2);
                     E += L * (s * m0 - sr);
-                    const int64_t ext = m0 - n0;
                     sumext += L * ext;
                     maxext = max(maxext, ext);
-                    viol += ext > alpha ? L : 0;
-                    kvviol += kv_sum > kv_cap ? L : 0;
-                    peakkv = max(peakkv, kv_sum);
-                    peakb = max(peakb, s);
-                    Tb += L;
-                    tok += s * L;
+                    viol += ext > alpha32 ? (int32_t)L : 0;
+                    kvviol += kv_over ? (int32_t)L : 0;
+                    Tb += (int32_t)L;
+                    tok += (int32_t)(s * L);
                 }
-                if (nxt > INT_MAX) { status = ISJL_ERR_STEP_LIMIT; break; }
-                k = (int32_t)nxt;
+                k = nxt;
             }
         }
     }
@@ -591,8 +599,17 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     __syncwarp();
 }
 
+// resident blocks per SM the register allocation is bounded for (measured
+// best on GB300 for the online sweep: 6 for the step kernel, 4 for the epoch one)
+#ifndef ISJL_SIM_MIN_BLOCKS_STEP
+#define ISJL_SIM_MIN_BLOCKS_STEP 6
+#endif
+#ifndef ISJL_SIM_MIN_BLOCKS_EPOCH
+#define ISJL_SIM_MIN_BLOCKS_EPOCH 4
+#endif
+
 template <int SPL, bool EPOCH>
-__global__ void __launch_bounds__(kSimWarpsPerBlock * 32)
+__global__ void __launch_bounds__(kSimWarpsPerBlock * 32, EPOCH ? ISJL_SIM_MIN_BLOCKS_EPOCH : ISJL_SIM_MIN_BLOCKS_STEP)
 sim_kernel(SimArgs A, int64_t n_tasks) {
     extern __shared__ __align__(16) int32_t smem[];
     const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
@@ -603,7 +620,9 @@ sim_kernel(SimArgs A, int64_t n_tasks) {
     S.shead = b + A.B;
     S.stail = b + 2 * A.B;
     S.slong = b + 3 * A.B;
-    S.pend0 = reinterpret_cast<uint32_t *>(b + 4 * A.B);
+    S.srem = b + 4 * A.B;
+    S.spsum = b + 5 * A.B;
+    S.pend0 = reinterpret_cast<uint32_t *>(b + 6 * A.B);
     S.pend1 = S.pend0 + A.words0;
     const int64_t gwarp = (int64_t)blockIdx.x * kSimWarpsPerBlock + wib;
     for (;;) {
@@ -659,9 +678,8 @@ int sim_resident_warps(int B, int n, bool epoch, int device) {
 }
 
 cudaError_t launch_sim(const SimArgs &args, bool epoch, int total_warps, cudaStream_t s) {
-    int bps = 0, sms = 0;
+    int bps = 0, sms = 0, dev = 0;
     size_t smem = 0;
-    int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     e = occupancy(args.B, args.n, epoch, dev, &bps, &sms, &smem);
