@@ -200,6 +200,38 @@ int32_t isjl_sim_last_launches(const isjl_sim *sim);
  * -1 on a CUDA error. */
 int32_t isjl_sim_kernel_times(const isjl_sim *sim, float *ms, int32_t cap);
 
+/* The sweep of isjl_sim_run_sweep without any allocation and without a
+ * handle.  The paper has no counterpart; this is a library service.
+ *
+ * For callers that cannot call cudaMalloc at the point of use: code running
+ * inside an allocator or memory pool that owns all device memory, processes
+ * under a fixed device-memory budget, and callers that must not let an
+ * allocation or free synchronize the device.  The workspace (derived lengths,
+ * sort arrays, plan links, work counter) lives in a fixed array of
+ * ISJL_NOALLOC_SCRATCH_BYTES bytes of device memory that every GPU loading
+ * this library holds until the process exits.  The caller passes the input
+ * arrays and the output buffers exactly as for isjl_sim_run_sweep (records
+ * required, start / completion optional, all device memory); no summaries are
+ * produced and device-side errors appear only in the records' status fields.
+ *
+ * cfg: as for isjl_sim_create (ISJL_FLAG_TIMING not accepted).  The first
+ * call with a given device current looks up the array's device address for
+ * that device; make that first call before any stream capture.  All calls
+ * share the one array and its contents persist between calls: calls whose
+ * GPU work overlaps (other streams, other threads) race and must be
+ * serialized by the caller.  Asynchronous on stream.
+ *
+ * Limit: the workspace needs 16 bytes per request (20 when
+ * n_per_instance > 4096), 40 bytes per instance, and n_per_instance * 16 bytes
+ * per block of the simulation kernel; fewer blocks run when the array cannot
+ * hold all resident ones.  That is about 3 to 4 million requests per call.
+ * Errors: INVALID_ARG (as isjl_sim_run_sweep, or the problem does not fit the
+ * fixed workspace), CUDA (symbol lookup or launch failure). */
+#define ISJL_NOALLOC_SCRATCH_BYTES (64u << 20)
+isjl_status isjl_sim_run_sweep_noalloc(const isjl_config *cfg, int32_t n_runs, const int32_t *policies,
+                                       const int32_t *deltas, int32_t kv_cap, const isjl_instances *in,
+                                       const isjl_outputs *out, void *stream);
+
 /* Static description of a status code (never NULL). */
 const char *isjl_status_string(isjl_status status);
 

@@ -62,7 +62,7 @@ assert ctypes.sizeof(isjl_record) == RECORD_DTYPE.itemsize == 192
 
 EXPORTS = ["isjl_sim_create", "isjl_sim_destroy", "isjl_sim_run", "isjl_sim_run_sweep",
            "isjl_sim_run_sweep_host", "isjl_sim_metrics", "isjl_sim_last_launches", "isjl_sim_kernel_times",
-           "isjl_status_string"]
+           "isjl_sim_run_sweep_noalloc", "isjl_status_string"]
 
 _lib = None
 
@@ -93,6 +93,9 @@ def lib():
         L.isjl_sim_last_launches.restype = i32
         L.isjl_sim_kernel_times.argtypes = [vp, ctypes.POINTER(ctypes.c_float), i32]
         L.isjl_sim_kernel_times.restype = i32
+        L.isjl_sim_run_sweep_noalloc.argtypes = [ctypes.POINTER(isjl_config), i32, p32, p32, i32,
+                                                 ctypes.POINTER(isjl_instances), ctypes.POINTER(isjl_outputs), vp]
+        L.isjl_sim_run_sweep_noalloc.restype = ctypes.c_int
         L.isjl_status_string.argtypes = [ctypes.c_int]
         L.isjl_status_string.restype = ctypes.c_char_p
         _lib = L
@@ -174,6 +177,25 @@ def isjl_sim_run_sweep_host(handle, policies, deltas, kv_cap, h_arrival, h_promp
     return lib().isjl_sim_run_sweep_host(handle, len(pol), pol, dl, int(kv_cap), h_arrival.data_ptr(),
                                          h_prompt.data_ptr(), h_output.data_ptr(), h_records.data_ptr(),
                                          _stream_ptr(stream))
+
+
+def isjl_sim_run_sweep_noalloc(n_instances, n_per_instance, B, policies, deltas, kv_cap, arrival, prompt,
+                               output, records, start=None, completion=None, c=0.0005, tau=1e-6, p0=0.002,
+                               max_steps=0, flags=FLAG_STEP_KERNEL, stream=None):
+    """Allocation-free sweep for callers that cannot allocate device memory at the
+    point of use (allocator-owned pools, fixed budgets, no-sync sections): the
+    library's workspace is a fixed device array shared by all calls, so calls
+    must not overlap on the GPU.  Device int32 tensors in, device buffers out;
+    returns the status code (no exception, no summaries)."""
+    cfg = isjl_config(int(n_instances), int(n_per_instance), int(B), float(c), float(tau), float(p0),
+                      int(max_steps), int(flags))
+    pol = _i32_array([_policy_code(p) for p in policies])
+    dl = _i32_array(deltas)
+    ins = isjl_instances(arrival.data_ptr(), prompt.data_ptr(), output.data_ptr())
+    outs = isjl_outputs(records.data_ptr(), start.data_ptr() if start is not None else None,
+                        completion.data_ptr() if completion is not None else None)
+    return lib().isjl_sim_run_sweep_noalloc(ctypes.byref(cfg), len(pol), pol, dl, int(kv_cap), ctypes.byref(ins),
+                                            ctypes.byref(outs), _stream_ptr(stream))
 
 
 def isjl_sim_metrics(handle, max_runs=MAX_RUNS):
