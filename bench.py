@@ -49,9 +49,10 @@ ALU_LANES_PER_SM = 128
 # violation, T_busy, token counter)
 OPS_PER_TOKEN_ADVANCE = 5
 OPS_PER_BATCH_STEP = 6
-# DRAM bytes (read + write) per launch of the simulation kernel, scaled from an
-# ncu capture of a 512-instance case of this workload; None until captured
-SIM_DRAM_BYTES_PER_LAUNCH = None
+# DRAM bytes (read + write) per launch of the step simulation kernel on the full
+# workload: 576.7 MB measured by ncu on the first 4,096 instances, scaled by
+# 10,000 / 4,096 (profiles/sim_kernel_step_online_delta_sweep_4096.md)
+SIM_DRAM_BYTES_PER_LAUNCH = 576.7e6 * 10_000 / 4_096
 
 
 def workload_config(kernel, wl, flush):
@@ -150,6 +151,19 @@ def dist_env():
     return world, rank, local
 
 
+def combine_ranks(t_ms, units, e2e_ms, dist=None, device="cpu"):
+    """Whole-job figures: the max over ranks of the timed milliseconds (and of
+    the e2e milliseconds) and the sum over ranks of the units processed."""
+    if dist is None:
+        return t_ms, units, e2e_ms
+    import torch
+    t = torch.tensor([t_ms, e2e_ms], dtype=torch.float64, device=device)
+    u = torch.tensor([units], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t[0]), float(u[0]), float(t[1])
+
+
 def reference_arm(args):
     world, rank, _ = dist_env()
     if rank != 0:
@@ -195,6 +209,7 @@ def main():
     ap.add_argument("--instances", type=int, default=0, help="use only the first N instances (profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-epoch", action="store_true", help="skip the event-driven kernel's extra measurement")
     args = ap.parse_args()
     if args.impl == "reference":
         return reference_arm(args)
@@ -247,29 +262,48 @@ def main():
         uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
     except Exception:
         uuid = None
+    def timed_steps(simr):
+        """K timed sweeps (L2 flushed before each, outside the events)."""
+        sim_ms = []
+        ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for k in range(args.steps):
+            flush.zero_()
+            ev0[k].record(stream)
+            simr.sweep_async(a, p, o, POLICIES, DELTAS, kv, per_request=True)
+            ev1[k].record(stream)
+            sim_ms.append(sim.isjl_sim_kernel_times(simr.handle)[2])   # waits for this step's events
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        wall_s = time.perf_counter() - t0
+        return [ev0[k].elapsed_time(ev1[k]) for k in range(args.steps)], sim_ms, wall_s
+
     sampler = ClockSampler(uuid)
     time.sleep(0.4)
-    step_ms, sim_ms = [], []
-    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
-    t_wall = time.perf_counter()
-    for k in range(args.steps):
-        flush.zero_()                      # evict L2 between timed steps (outside the events)
-        ev0[k].record(stream)
-        S.sweep_async(a, p, o, POLICIES, DELTAS, kv, per_request=True)
-        ev1[k].record(stream)
-        kt = sim.isjl_sim_kernel_times(S.handle)   # waits for this step's events
-        sim_ms.append(kt[2])
-    torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
-    wall = time.perf_counter() - t_wall
+    step_ms, sim_ms, wall = timed_steps(S)
     clocks = sampler.stop()
-    step_ms = [ev0[k].elapsed_time(ev1[k]) for k in range(args.steps)]
     t_ms = sum(step_ms)
+
+    # the other kernel variant on the same inputs (same results), for comparison
+    other = None
+    if not args.no_epoch:
+        S2 = sim.Simulator(n_inst, wl.n_per_instance, B, wl.c, wl.tau, wl.p0, epoch=not epoch, timing=True)
+        for _ in range(max(args.warmup, 1)):
+            S2.sweep_async(a, p, o, POLICIES, DELTAS, kv, per_request=True)
+        st2, summ2 = sim.isjl_sim_metrics(S2.handle)
+        busy2 = sum(summ2[i].T_busy for i in range(len(POLICIES)))
+        if st2 != 0 or busy2 != busy_per_step:
+            raise RuntimeError("kernel variants disagree")
+        step2, sim2, _ = timed_steps(S2)
+        other = {"kernel": "step" if epoch else "epoch",
+                 "value": busy_per_step * args.steps / (sum(step2) / 1e3),
+                 "ms_per_step": sum(step2) / args.steps, "sim_ms_per_launch": sum(sim2) / len(sim2)}
+        S2.close()
 
     # e2e through the host-memory entry point: H2D of the inputs, sweep, D2H of the records
     e2e = None
@@ -290,15 +324,7 @@ def main():
 
     # max over ranks, sum of units
     units = float(busy_per_step * args.steps)
-    if dist:
-        t = torch.tensor([t_ms, units, e2e["ms"] if e2e else 0.0], dtype=torch.float64, device="cuda")
-        tmax = t.clone()
-        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
-        tsum = t.clone()
-        dist.all_reduce(tsum, op=dist.ReduceOp.SUM)
-        t_ms_all, units_all, e2e_ms_all = float(tmax[0]), float(tsum[1]), float(tmax[2])
-    else:
-        t_ms_all, units_all, e2e_ms_all = t_ms, units, (e2e["ms"] if e2e else 0.0)
+    t_ms_all, units_all, e2e_ms_all = combine_ranks(t_ms, units, e2e["ms"] if e2e else 0.0, dist, "cuda")
 
     if rank != 0:
         if dist:
@@ -320,7 +346,8 @@ def main():
         ops = OPS_PER_TOKEN_ADVANCE * tok_per_step + OPS_PER_BATCH_STEP * busy_per_step
         achieved = ops / (sim_avg_ms / 1e3) / 1e12
         roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s",
-                    "frac": achieved / peak_tops, "traffic": SIM_DRAM_BYTES_PER_LAUNCH,
+                    "frac": achieved / peak_tops,
+                    "traffic": SIM_DRAM_BYTES_PER_LAUNCH if n_inst == wl.n_instances else None,
                     "kernel": "sim_kernel (step)", "ops_per_launch": ops,
                     "peak_basis": f"{sms} SMs x {ALU_LANES_PER_SM} int32 lanes x {sm_mhz:.0f} MHz (median SM clock "
                                   "sampled during the timed steps)",
@@ -328,7 +355,7 @@ def main():
 
     cpu = None
     if pool is not None:
-        per_core = 8
+        per_core = 40          # about 20 s of single-core oracle work in total
         sample_n = min(n_inst, cores * per_core)
         tb, tok, dt = oracle_timed(a_h[:sample_n], p_h[:sample_n], o_h[:sample_n], B, kv, cores, pool)
         pool.close()
@@ -353,6 +380,7 @@ def main():
         "instances_per_s": world * n_inst * len(POLICIES) * args.steps / (t_ms_all / 1e3),
         "token_advances_per_s": tok_per_step * world * args.steps / (t_ms_all / 1e3),
         "kernel_ms": {"sim": sim_avg_ms},
+        "other_kernel": other,
         "wall_s": wall,
     }
     print(json.dumps(line), flush=True)

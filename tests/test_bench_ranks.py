@@ -1,0 +1,50 @@
+"""Multi-rank host logic of bench.py on CPU (gloo, world size 2): each rank
+simulates an independent replica of the workload, and the whole-job figures
+are the max of the timings and the sum of the units over ranks."""
+import os
+import socket
+
+import numpy as np
+import pytest
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, out):
+    import torch.distributed as dist
+    import bench
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    t, u, e = bench.combine_ranks(10.0 + rank, 100.0 * (rank + 1), 20.0 - rank, dist, "cpu")
+    out[rank] = (t, u, e)
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_combine_ranks_gloo_world2():
+    import torch.multiprocessing as mp
+    port = _free_port()
+    mgr = mp.Manager()
+    out = mgr.dict()
+    mp.spawn(_worker, args=(2, port, out), nprocs=2, join=True)
+    for r in range(2):
+        assert out[r] == (11.0, 300.0, 20.0)
+
+
+def test_single_rank_passthrough():
+    import bench
+    assert bench.combine_ranks(5.0, 7.0, 9.0, None) == (5.0, 7.0, 9.0)
+
+
+def test_rank_replicas_are_independent_instances():
+    from paper_2608_02244_gb300 import workloads as W
+    a0, p0, o0 = W.generate(3, 2, replica=0)
+    a1, p1, o1 = W.generate(3, 2, replica=1)
+    assert not np.array_equal(p0, p1) and a0.shape == a1.shape
+    a0b, _, _ = W.generate(3, 2)
+    np.testing.assert_array_equal(a0, a0b)
