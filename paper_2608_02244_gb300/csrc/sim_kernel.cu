@@ -71,6 +71,11 @@ __device__ __forceinline__ int highest_worker(uint32_t m, int lane) {
     return __reduce_max_sync(kFull, v);
 }
 
+// acc += a * b into a 64-bit accumulator with one wide multiply-add
+__device__ __forceinline__ void mad_wide(int64_t &acc, uint32_t a, uint32_t b) {
+    asm("mad.wide.u32 %0, %1, %2, %0;" : "+l"(acc) : "r"(a), "r"(b));
+}
+
 __device__ __forceinline__ int64_t warp_sum64(int64_t v) {
 #pragma unroll
     for (int s = 16; s > 0; s >>= 1) v += __shfl_xor_sync(kFull, v, s);
@@ -177,6 +182,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 #pragma unroll
         for (int r = 0; r < SPL; ++r) { sa[r] = kIdle; sc[r] = INT_MAX; }
         uint32_t busy = 0u, resv = 0u;
+        uint32_t lhead = 0u;    // worker's next plan entry is its long job o_j (waits for o_1)
         int32_t lane_cmin = INT_MAX;                 // earliest completion among this lane's workers
         int32_t lane_smin = INT_MAX, lane_smax = INT_MIN;   // start range (epoch kernel)
         const int nrow = (B - lane + 31) >> 5;       // rows holding a valid worker for this lane
@@ -185,8 +191,19 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 
         int32_t k = 0, rel = 0, fcfs = 0, done = 0, run_cnt = 0, pend = 0;
         int64_t kv_sum = 0, sum_st = 0;
+        // the next 32 unreleased requests (from win_base): arrival and sorted position, per lane
+        int32_t win_base = 0, win_a = INT_MAX, win_p = 0;
+        auto load_window = [&]() {
+            const int i = win_base + lane;
+            win_a = i < n ? arr[i] : INT_MAX;
+            win_p = (i < n && policy != ISJL_POLICY_FCFS) ? posof[i] : 0;
+        };
+        load_window();
         // uniform caches, changed only at events
-        int32_t next_arr = n > 0 ? arr[0] : INT_MAX;   // arrival of the next unreleased request
+        int32_t next_arr = __shfl_sync(kFull, win_a, 0);   // arrival of the next unreleased request
+        int32_t hp = INT_MAX, ho = 0, ho_pos = -1;     // longest pending position and its o (LJF / ISJL)
+        bool hvalid = true;                            // hp is current (else recompute from the bitset)
+        int32_t fo = -1;                               // o of the FCFS head (-1: not loaded)
         int32_t cmin = INT_MAX;                        // earliest completion step of the running set
         int32_t smin = INT_MAX, smax = INT_MIN;        // start range of the running set (epoch kernel)
         int32_t kv_over = 0;                           // reserved KV above the cap (never, by construction)
@@ -238,14 +255,14 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         auto retire = [&](int32_t c) {
             uint32_t fm = 0u;
             int nf = 0, of = 0;
-            int64_t sf = 0;
+            unsigned sf = 0u;   // sum of (start - (c - 65536)) over finishing requests (epoch kernel)
 #pragma unroll
             for (int r = 0; r < SPL; ++r) {
                 if ((busy >> r & 1u) && sc[r] == c) {
                     fm |= 1u << r;
                     nf++;
                     of += EPOCH ? sc[r] - sa[r] : sa[r];
-                    if (EPOCH) sf += sa[r];
+                    if (EPOCH) sf += (unsigned)(sa[r] - (c - 65536));
                     if (co_out) co_out[S.sjob[(r << 5) + lane]] = c;
                     sc[r] = INT_MAX;
                     if (!EPOCH) sa[r] = kIdle + c - 1;   // sentinel of the step just served
@@ -255,7 +272,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (fm) recompute_lane();
             nf = (int)__reduce_add_sync(kFull, (unsigned)nf);
             of = (int)__reduce_add_sync(kFull, (unsigned)of);
-            if (EPOCH) sum_st -= warp_sum64(sf);
+            if (EPOCH)   // starts are within 65535 steps of c, so the offsets fit 32 bits
+                sum_st -= (int64_t)__reduce_add_sync(kFull, sf) + (int64_t)nf * (c - 65536);
             done += nf;
             run_cnt -= nf;
             kv_sum -= of;
@@ -276,6 +294,41 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 #pragma unroll
             for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = max(m, sa[r]);
             return (int64_t)__reduce_max_sync(kFull, m);
+        };
+
+        auto release = [&]() {
+            for (;;) {
+                // released: window lanes at or after rel whose arrival is <= k (a prefix)
+                const bool ok = win_base + lane >= rel && win_a <= k;
+                const unsigned b = __ballot_sync(kFull, ok);
+                if (policy != ISJL_POLICY_FCFS) {
+                    if (ok) {
+                        atomicOr(&S.pend0[win_p >> 5], 1u << (win_p & 31));
+                        atomicOr(&S.pend1[win_p >> 10], 1u << ((win_p >> 5) & 31));
+                    }
+                    if (hvalid) hp = min(hp, __reduce_min_sync(kFull, ok ? win_p : INT_MAX));
+                }
+                const int c = __popc(b);
+                rel += c;
+                pend += c;
+                if (rel < win_base + 32 || win_base + 32 >= n) break;
+                win_base += 32;                           // window used up: load the next 32
+                load_window();
+            }
+            __syncwarp();
+            next_arr = rel < n ? __shfl_sync(kFull, win_a, (rel - win_base) & 31) : INT_MAX;
+        };
+        // longest pending position (INT_MAX if none) and its length
+        auto head = [&]() -> int {
+            if (!hvalid) { hp = bs_next(S, words0, words1, 0, lane); hvalid = true; }
+            if (hp < n && ho_pos != hp) { ho = osrt[hp]; ho_pos = hp; }
+            return hp;
+        };
+        // remove the head position p (the longest pending request)
+        auto pop_head = [&](int p) {
+            bs_clear(S, p, lane);
+            pend--;
+            hp = bs_next(S, words0, words1, p + 1, lane);   // nothing pending below p
         };
 
         // ISJL Phase ONE at a stage start (Algorithm 2 with beta = alpha)
@@ -373,40 +426,48 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             mx = __reduce_max_sync(kFull, mx);
             d1 = (int32_t)min(max((int64_t)mx - alpha, (int64_t)0), alpha);
             resv = 0u;
+            lhead = 0u;
 #pragma unroll
             for (int r = 0; r < SPL; ++r) {
                 const int w = (r << 5) + lane;
                 if (w < B && S.shead[w] >= 0) resv |= 1u << r;
+                if (w >= 1 && w < nl && S.shead[w] == S.slong[w]) lhead |= 1u << r;
             }
             L1_started = false;
             nlong = nl;
+            hvalid = false;                                // Phase ONE removed queued requests
+            // spsum now caches the length of each worker's next plan entry
+            for (int w = lane; w < B; w += 32) {
+                const int e = S.shead[w];
+                S.spsum[w] = e >= 0 ? oarr[e] : 0;
+            }
+            __syncwarp();
         };
 
         auto admit = [&]() {
             if (policy == ISJL_POLICY_FCFS) {
                 // arrival order; the first request that does not fit ends the step
                 while (run_cnt < B && fcfs < rel) {
-                    const int oe = oarr[fcfs];
-                    if (kv_sum + oe > kv_cap) break;
+                    if (fo < 0) fo = oarr[fcfs];
+                    if (kv_sum + fo > kv_cap) break;
                     const int w = lowest_worker(vmask & ~busy, lane);
                     if (w < 0) { broken = true; return; }
-                    start(fcfs, oe, w);
+                    start(fcfs, fo, w);
                     fcfs++;
+                    fo = -1;
                 }
             } else if (policy == ISJL_POLICY_LJF) {
                 // static batch of the longest released requests when nothing runs
                 if (run_cnt != 0) return;
-                int p = -1;
                 while (run_cnt < B && pend > 0) {
-                    p = bs_next(S, words0, words1, p + 1, lane);
+                    const int p = head();
                     if (p >= n) { broken = true; return; }
-                    const int oe = osrt[p];
-                    if (kv_sum + oe > kv_cap) break;
+                    if (kv_sum + ho > kv_cap) break;
                     const int e = perm[p];
                     const int w = lowest_worker(vmask & ~busy, lane);
                     if (w < 0) { broken = true; return; }
-                    bs_clear(S, p, lane);
-                    pend--;
+                    const int oe = ho;
+                    pop_head(p);
                     start(e, oe, w);
                 }
             } else {
@@ -415,8 +476,14 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (broken) return;
                 bool stop = amax_now() > alpha;                  // the gate A_max(k) <= alpha
                 if (!stop && plan_left > 0) {
-                    // plan starts, workers in order
+                    // plan starts, workers in order; entries that must wait (o_1's
+                    // delay, o_j before o_1) are filtered out up front
                     uint32_t cand = resv & ~busy;
+                    if (!L1_started) {
+                        cand &= ~lhead;
+                        const bool over = ((int64_t)k >= (int64_t)t0 + d1) || (k > t0 && nothing_runs);
+                        if (!over && lane == 0) cand &= ~1u;        // worker 0 holds o_1
+                    }
                     for (;;) {
                         const int w = lowest_worker(cand, lane);
                         if (w < 0) break;
@@ -427,31 +494,40 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                             if (!over) continue;                 // o_1 still delayed
                         }
                         if (w >= 1 && w < nlong && e == S.slong[w] && !L1_started) continue;  // o_j after o_1
-                        const int oe = oarr[e];
+                        const int oe = S.spsum[w];                 // o of the worker's next entry
                         if (kv_sum + oe > kv_cap) { stop = true; break; }
                         const int nx = pnext[e];
                         __syncwarp();
-                        if (lane == 0) { S.shead[w] = nx; if (nx < 0) S.stail[w] = kNone; }
+                        if (lane == 0) {
+                            S.shead[w] = nx;
+                            if (nx < 0) S.stail[w] = kNone; else S.spsum[w] = oarr[nx];
+                        }
                         __syncwarp();
-                        if (nx < 0 && lane == (w & 31)) resv &= ~(1u << (w >> 5));
+                        if (lane == (w & 31)) {
+                            const uint32_t bit = 1u << (w >> 5);
+                            if (nx < 0) resv &= ~bit;
+                            if (w >= 1 && w < nlong && nx >= 0 && nx == S.slong[w]) lhead |= bit;
+                            else lhead &= ~bit;
+                        }
                         plan_left--;
-                        if (e == L1) L1_started = true;
+                        if (e == L1) {
+                            L1_started = true;
+                            cand |= resv & ~busy & lhead;            // the o_j may start now
+                        }
                         start(e, oe, w);
                     }
                 }
                 if (!stop) {
                     // Phase TWO: longest released request onto a free worker
-                    int p = -1;
                     while (pend > 0) {
                         const int w = lowest_worker(vmask & ~busy & ~resv, lane);
                         if (w < 0) break;
-                        p = bs_next(S, words0, words1, p + 1, lane);
+                        const int p = head();
                         if (p >= n) { broken = true; return; }
-                        const int oe = osrt[p];
-                        if (kv_sum + oe > kv_cap) break;
+                        if (kv_sum + ho > kv_cap) break;
                         const int e = perm[p];
-                        bs_clear(S, p, lane);
-                        pend--;
+                        const int oe = ho;
+                        pop_head(p);
                         start(e, oe, w);
                     }
                 }
@@ -459,25 +535,6 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         };
 
         // release every request with A_i <= k (a prefix: arrivals are non-decreasing)
-        auto release = [&]() {
-            for (;;) {
-                const int i = rel + lane;
-                const bool ok = i < n && arr[i] <= k;
-                const unsigned b = __ballot_sync(kFull, ok);
-                if (ok && policy != ISJL_POLICY_FCFS) {
-                    const int p = posof[i];
-                    atomicOr(&S.pend0[p >> 5], 1u << (p & 31));
-                    atomicOr(&S.pend1[p >> 10], 1u << ((p >> 5) & 31));
-                }
-                const int c = __popc(b);
-                rel += c;
-                pend += c;
-                if (c < 32) break;
-            }
-            __syncwarp();
-            next_arr = rel < n ? arr[rel] : INT_MAX;
-        };
-
         if (!EPOCH) {
             // ---------------------------------------------------- step kernel
             int32_t next_check = 0;   // the next step needing release / admission / the guard
@@ -512,9 +569,9 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     sm = __reduce_add_sync(kFull, sm);
                     sm -= idle_slots * (unsigned)(kIdle + k);     // idle slots each added kIdle + k
                     const int ext = mx - (int)mn;
-                    W += (int64_t)run_cnt * mx;                   // |S| max r
-                    R += (int64_t)(int32_t)sm;                    // sum r
-                    sumext += ext;
+                    mad_wide(W, (uint32_t)run_cnt, (uint32_t)mx); // |S| max r
+                    mad_wide(R, sm, 1u);                          // sum r (>= 0)
+                    mad_wide(sumext, (uint32_t)ext, 1u);
                     maxext = max(maxext, ext);
                     viol += ext > alpha32;
                     Tb++;
@@ -600,9 +657,9 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 }
 
 // resident blocks per SM the register allocation is bounded for (measured
-// best on GB300 for the online sweep: 6 for the step kernel, 4 for the epoch one)
+// best on GB300 for the online sweep: 4 for both variants)
 #ifndef ISJL_SIM_MIN_BLOCKS_STEP
-#define ISJL_SIM_MIN_BLOCKS_STEP 6
+#define ISJL_SIM_MIN_BLOCKS_STEP 4
 #endif
 #ifndef ISJL_SIM_MIN_BLOCKS_EPOCH
 #define ISJL_SIM_MIN_BLOCKS_EPOCH 4
