@@ -81,11 +81,16 @@ typedef struct {
     uint32_t flags;          /* ISJL_FLAG_* */
 } isjl_config;
 
-/* Inputs: three device arrays of n_instances * n_per_instance int32 each. */
+/* Inputs: three device arrays of n_instances * n_per_instance int32 each,
+ * plus an optional per-instance request count for ragged batches. */
 typedef struct {
     const int32_t *arrival;  /* release step A_i >= 0, non-decreasing within an instance */
     const int32_t *prompt;   /* prompt tokens >= 0 */
     const int32_t *output;   /* output tokens >= 0; o_i = prompt + output must be 1..ISJL_MAX_LEN */
+    const int32_t *count;    /* device, n_instances entries or NULL: instance i uses its first
+                                count[i] slots (0..n_per_instance; 0 = an empty instance, all
+                                counters 0); NULL = every instance uses all n_per_instance.  A
+                                count outside 0..n_per_instance makes that instance INVALID_ARG. */
 } isjl_instances;
 
 /* One result record per (run, instance).  Integers are exact; the doubles
@@ -114,7 +119,7 @@ typedef struct {
     double revenue;          /* p0 * O */
     double profit;           /* revenue - cost */
     double throughput;       /* O / T_make, tokens per step */
-    double ael;              /* sum_completion / n */
+    double ael;              /* sum_completion / n (0 for an empty instance) */
 } isjl_record;
 
 /* Where results go.  records: device, n_runs * n_instances entries,

@@ -267,9 +267,10 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
                int32_t *start_out, int32_t *compl_out, or_record *rec)
 {
     memset(rec, 0, sizeof(*rec));
-    if (n < 1 || B < 1 || delta < 0 || kv_cap < 1 || policy < 0 || policy > 2 || !arrival || !prompt || !output) {
+    if (n < 0 || B < 1 || delta < 0 || kv_cap < 1 || policy < 0 || policy > 2 || (n > 0 && (!arrival || !prompt || !output))) {
         rec->status = OR_INVALID_ARG; return OR_INVALID_ARG;
     }
+    if (n == 0) return OR_OK;   /* an empty instance: nothing runs, every counter is 0 */
     for (int i = 0; i < n; ++i) {
         if (arrival[i] < 0 || prompt[i] < 0 || output[i] < 0 || (i > 0 && arrival[i] < arrival[i - 1])) {
             rec->status = OR_INVALID_ARG; return OR_INVALID_ARG;

@@ -63,13 +63,40 @@ def _ptr(a):
 
 
 def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p0=0.002,
-        max_steps=0, per_request=True):
+        max_steps=0, per_request=True, counts=None):
     """Simulate every instance (row) under one policy and budget.
 
     Returns (records, start, completion); records is a structured array with
     one entry per instance (fields RECORD_DTYPE), start/completion are int32
     arrays shaped like ``arrival`` (None when per_request is False).
+    ``counts`` (optional, one per row) limits instance i to its first
+    counts[i] requests (ragged batches); the rest stay -1.
     """
+    if counts is not None:
+        a, p, o = (np.atleast_2d(_i32(x)) for x in (arrival, prompt, output))
+        recs, sts, cos = [], [], []
+        for i, m in enumerate(np.asarray(counts)):
+            m = int(m)
+            if m < 0 or m > a.shape[1]:            # a count outside 0..n: invalid instance
+                r = np.zeros(1, RECORD_DTYPE)
+                r["status"] = 1
+                recs.append(r)
+                if per_request:
+                    sts.append(np.full((1, a.shape[1]), -1, np.int32))
+                    cos.append(np.full((1, a.shape[1]), -1, np.int32))
+                continue
+            r, st, co = run(policy, B, delta, kv_cap, a[i:i + 1, :m], p[i:i + 1, :m], o[i:i + 1, :m], c, tau, p0,
+                            max_steps, per_request)
+            recs.append(r)
+            if per_request:
+                row = np.full((1, a.shape[1]), -1, np.int32)
+                rc = row.copy()
+                row[0, :m] = st[0, :m] if m else row[0, :0]
+                rc[0, :m] = co[0, :m] if m else rc[0, :0]
+                sts.append(row)
+                cos.append(rc)
+        rec = np.concatenate(recs)
+        return rec, (np.concatenate(sts) if per_request else None), (np.concatenate(cos) if per_request else None)
     a, p, o = _i32(arrival), _i32(prompt), _i32(output)
     squeeze = a.ndim == 1
     if squeeze:

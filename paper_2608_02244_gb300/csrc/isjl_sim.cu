@@ -138,11 +138,11 @@ isjl_status isjl_sim_run_sweep(isjl_sim *s, int32_t n_runs, const int32_t *polic
     if (cudaMemsetAsync(s->d_counter, 0, sizeof(int32_t), st) != cudaSuccess ||
         cudaMemsetAsync(s->d_status, 0, sizeof(int32_t), st) != cudaSuccess || !mark(0))
         return ISJL_ERR_CUDA;
-    if (isjl::launch_derive(in->arrival, in->prompt, in->output, s->d_o, s->d_inst, c.n_instances,
+    if (isjl::launch_derive(in->arrival, in->prompt, in->output, in->count, s->d_o, s->d_inst, c.n_instances,
                             c.n_per_instance, st) != cudaSuccess || !mark(1))
         return ISJL_ERR_CUDA;
     s->last_launches++;
-    if (isjl::launch_sort(s->d_o, s->d_perm, s->d_osorted, s->d_posof, s->d_tmp, c.n_instances,
+    if (isjl::launch_sort(s->d_o, s->d_inst, s->d_perm, s->d_osorted, s->d_posof, s->d_tmp, c.n_instances,
                           c.n_per_instance, st) != cudaSuccess || !mark(2))
         return ISJL_ERR_CUDA;
     s->last_launches++;

@@ -105,10 +105,10 @@ extern "C" isjl_status isjl_sim_run_sweep_noalloc(const isjl_config *cfg, int32_
 
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (cudaMemsetAsync(d_ctr, 0, 2 * sizeof(int32_t), st) != cudaSuccess) return ISJL_ERR_CUDA;
-    if (isjl::launch_derive(in->arrival, in->prompt, in->output, d_o, d_inst, cfg->n_instances, n, st) !=
+    if (isjl::launch_derive(in->arrival, in->prompt, in->output, in->count, d_o, d_inst, cfg->n_instances, n, st) !=
         cudaSuccess)
         return ISJL_ERR_CUDA;
-    if (isjl::launch_sort(d_o, d_perm, d_os, d_pos, d_tmp, cfg->n_instances, n, st) != cudaSuccess)
+    if (isjl::launch_sort(d_o, d_inst, d_perm, d_os, d_pos, d_tmp, cfg->n_instances, n, st) != cudaSuccess)
         return ISJL_ERR_CUDA;
 
     isjl::SimArgs a;

@@ -36,10 +36,13 @@ __device__ __forceinline__ T warp_max(T v) {
 // one block per instance
 __global__ void __launch_bounds__(kDeriveThreads)
 derive_kernel(const int32_t *__restrict__ arrival, const int32_t *__restrict__ prompt,
-              const int32_t *__restrict__ output, int32_t *__restrict__ o, InstStats *inst, int32_t n) {
-    const int64_t base = (int64_t)blockIdx.x * n;
+              const int32_t *__restrict__ output, const int32_t *__restrict__ count, int32_t *__restrict__ o,
+              InstStats *inst, int32_t n_slots) {
+    const int64_t base = (int64_t)blockIdx.x * n_slots;
     int64_t O = 0, Q = 0, sumA = 0;
     int32_t maxo = 0, maxA = 0, invalid = 0, infeasible = 0;
+    int32_t n = count ? count[blockIdx.x] : n_slots;
+    if (n < 0 || n > n_slots) { invalid = 1; n = 0; }
     for (int i = threadIdx.x; i < n; i += kDeriveThreads) {
         const int32_t a = arrival[base + i], p = prompt[base + i], q = output[base + i];
         const int64_t oi = (int64_t)p + q;
@@ -72,6 +75,7 @@ derive_kernel(const int32_t *__restrict__ arrival, const int32_t *__restrict__ p
             invalid |= s32[2][w]; infeasible |= s32[3][w];
         }
         st.status = invalid ? ISJL_ERR_INVALID_ARG : (infeasible ? ISJL_ERR_INFEASIBLE : ISJL_OK);
+        st.n = n;
         inst[blockIdx.x] = st;
     }
 }
@@ -83,10 +87,11 @@ __device__ __forceinline__ uint32_t len_key(int32_t o) {   // larger o sorts fir
 
 // n <= 4096: keys (65535 - o) << 16 | index, bitonic sort in shared memory
 __global__ void __launch_bounds__(kSortThreads)
-sort_small_kernel(const int32_t *__restrict__ o, int32_t *__restrict__ perm, int32_t *__restrict__ osorted,
-                  int32_t *__restrict__ posof, int32_t n, int32_t npow2) {
+sort_small_kernel(const int32_t *__restrict__ o, const InstStats *__restrict__ inst, int32_t *__restrict__ perm,
+                  int32_t *__restrict__ osorted, int32_t *__restrict__ posof, int32_t n_slots, int32_t npow2) {
     extern __shared__ uint32_t key[];
-    const int64_t base = (int64_t)blockIdx.x * n;
+    const int64_t base = (int64_t)blockIdx.x * n_slots;
+    const int32_t n = inst[blockIdx.x].n;
     for (int t = threadIdx.x; t < npow2; t += kSortThreads)
         key[t] = t < n ? (len_key(o[base + t]) << 16) | (uint32_t)t : 0xffffffffu;
     for (int size = 2; size <= npow2; size <<= 1) {
@@ -118,11 +123,13 @@ sort_small_kernel(const int32_t *__restrict__ o, int32_t *__restrict__ perm, int
 constexpr int kCntStride = kRadixThreads + 1;
 
 __global__ void __launch_bounds__(kRadixThreads)
-sort_radix_kernel(const int32_t *__restrict__ o, int32_t *__restrict__ perm, int32_t *__restrict__ osorted,
-                  int32_t *__restrict__ posof, int32_t *__restrict__ tmp, int32_t n) {
+sort_radix_kernel(const int32_t *__restrict__ o, const InstStats *__restrict__ inst, int32_t *__restrict__ perm,
+                  int32_t *__restrict__ osorted, int32_t *__restrict__ posof, int32_t *__restrict__ tmp,
+                  int32_t n_slots) {
     extern __shared__ uint32_t cnt[];             // [256][kCntStride]
     __shared__ uint32_t dbase[256];
-    const int64_t base = (int64_t)blockIdx.x * n;
+    const int64_t base = (int64_t)blockIdx.x * n_slots;
+    const int32_t n = inst[blockIdx.x].n;
     const int tid = threadIdx.x;
     const int chunk = (n + kRadixThreads - 1) / kRadixThreads;
     const int lo = min(n, tid * chunk), hi = min(n, lo + chunk);
@@ -237,24 +244,25 @@ summarize_kernel(const isjl_record *__restrict__ rec, int64_t n_inst, RunList ru
 }  // namespace
 
 cudaError_t launch_derive(const int32_t *arrival, const int32_t *prompt, const int32_t *output,
-                          int32_t *o, InstStats *inst, int64_t n_inst, int32_t n, cudaStream_t s) {
-    derive_kernel<<<(unsigned)n_inst, kDeriveThreads, 0, s>>>(arrival, prompt, output, o, inst, n);
+                          const int32_t *count, int32_t *o, InstStats *inst, int64_t n_inst, int32_t n,
+                          cudaStream_t s) {
+    derive_kernel<<<(unsigned)n_inst, kDeriveThreads, 0, s>>>(arrival, prompt, output, count, o, inst, n);
     return cudaGetLastError();
 }
 
-cudaError_t launch_sort(const int32_t *o, int32_t *perm, int32_t *osorted, int32_t *posof,
+cudaError_t launch_sort(const int32_t *o, const InstStats *inst, int32_t *perm, int32_t *osorted, int32_t *posof,
                         int32_t *tmp, int64_t n_inst, int32_t n, cudaStream_t s) {
     if (n <= kSortSmallMax) {
         int npow2 = 1;
         while (npow2 < n) npow2 <<= 1;
-        sort_small_kernel<<<(unsigned)n_inst, kSortThreads, npow2 * sizeof(uint32_t), s>>>(o, perm, osorted, posof,
-                                                                                         n, npow2);
+        sort_small_kernel<<<(unsigned)n_inst, kSortThreads, npow2 * sizeof(uint32_t), s>>>(o, inst, perm, osorted,
+                                                                                         posof, n, npow2);
         return cudaGetLastError();
     }
     const size_t smem = 256 * kCntStride * sizeof(uint32_t);
     cudaError_t e = cudaFuncSetAttribute(sort_radix_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    sort_radix_kernel<<<(unsigned)n_inst, kRadixThreads, smem, s>>>(o, perm, osorted, posof, tmp, n);
+    sort_radix_kernel<<<(unsigned)n_inst, kRadixThreads, smem, s>>>(o, inst, perm, osorted, posof, tmp, n);
     return cudaGetLastError();
 }
 

@@ -23,7 +23,7 @@ struct InstStats {
     int32_t maxo;     // largest o_i
     int32_t maxA;     // largest arrival
     int32_t status;   // ISJL_OK, ISJL_ERR_INVALID_ARG or ISJL_ERR_INFEASIBLE (o_i < 1)
-    int32_t pad;
+    int32_t n;        // requests of this instance (its first n slots)
 };
 
 // (policy, delta) list of one sweep, passed by value to the kernel.
@@ -59,8 +59,9 @@ struct SimArgs {
 
 // host-side launchers (defined in the .cu files)
 cudaError_t launch_derive(const int32_t *arrival, const int32_t *prompt, const int32_t *output,
-                          int32_t *o, InstStats *inst, int64_t n_inst, int32_t n, cudaStream_t s);
-cudaError_t launch_sort(const int32_t *o, int32_t *perm, int32_t *osorted, int32_t *posof,
+                          const int32_t *count, int32_t *o, InstStats *inst, int64_t n_inst, int32_t n,
+                          cudaStream_t s);
+cudaError_t launch_sort(const int32_t *o, const InstStats *inst, int32_t *perm, int32_t *osorted, int32_t *posof,
                         int32_t *tmp, int64_t n_inst, int32_t n, cudaStream_t s);
 cudaError_t launch_sim(const SimArgs &args, bool epoch, int total_warps, cudaStream_t s);
 cudaError_t launch_summarize(const isjl_record *records, int64_t n_inst, int32_t n_runs,

@@ -144,8 +144,10 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                                          int64_t task) {
     const int64_t inst = task / A.n_runs;
     const int run = (int)(task % A.n_runs);
-    const int n = A.n, B = A.B;
-    const int64_t base = inst * (int64_t)n;
+    const int n_slots = A.n, B = A.B;
+    const int64_t base = inst * (int64_t)n_slots;
+    const InstStats is = A.inst[inst];
+    const int n = is.n;                             // requests of this instance (<= n_slots)
     const int policy = A.runs.policy[run];
     const int64_t alpha = A.runs.delta[run];
     const int64_t kv_cap = A.kv_cap;
@@ -154,12 +156,11 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     const int32_t *__restrict__ perm = A.perm + base;
     const int32_t *__restrict__ osrt = A.osorted + base;
     const int32_t *__restrict__ posof = A.posof + base;
-    int32_t *pnext = A.plan_next + gwarp * (int64_t)n;
-    const int64_t out_off = (int64_t)run * A.n_inst * n + base;
+    int32_t *pnext = A.plan_next + gwarp * (int64_t)n_slots;
+    const int64_t out_off = (int64_t)run * A.n_inst * n_slots + base;
     int32_t *st_out = A.start_out ? A.start_out + out_off : nullptr;
     int32_t *co_out = A.compl_out ? A.compl_out + out_off : nullptr;
-    const InstStats is = A.inst[inst];
-    const int words0 = A.words0, words1 = A.words1;
+    const int words0 = (n + 31) >> 5, words1 = (words0 + 31) >> 5;
 
     int64_t status = is.status;
     if (status == ISJL_OK && (int64_t)is.maxo > kv_cap) status = ISJL_ERR_INFEASIBLE;
@@ -170,7 +171,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     int64_t W = 0, R = 0, E = 0, sumc = 0, sumext = 0, peakkv = 0;
     int32_t Tb = 0, tok = 0, maxext = 0, viol = 0, peakb = 0, Tmake = 0, kvviol = 0;
 
-    if (status == ISJL_OK) {
+    if (status == ISJL_OK && n > 0) {
         for (int w = lane; w < words0; w += 32) S.pend0[w] = 0u;
         for (int w = lane; w < words1; w += 32) S.pend1[w] = 0u;
         for (int w = lane; w < B; w += 32) { S.shead[w] = kNone; S.stail[w] = kNone; S.slong[w] = kNone; }
@@ -648,7 +649,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             R.revenue = __dmul_rn(A.p0, (double)is.O);
             R.profit = __dsub_rn(R.revenue, R.cost);
             R.throughput = Tmake > 0 ? __ddiv_rn((double)is.O, (double)Tmake) : 0.0;
-            R.ael = __ddiv_rn((double)sumc, (double)n);
+            R.ael = n > 0 ? __ddiv_rn((double)sumc, (double)n) : 0.0;
         }
         A.records[(int64_t)run * A.n_inst + inst] = R;
         if (status != ISJL_OK) atomicCAS(A.dev_status, 0, (int32_t)status);

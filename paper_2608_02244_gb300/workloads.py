@@ -43,6 +43,7 @@ class Workload:
     deltas: tuple       # ISJL fairness budgets
     policies: tuple = ("fcfs", "ljf", "isjl")
     online: bool = False
+    ragged: bool = False  # instances use a variable number of their slots (see counts)
     note: str = ""
     c: float = 0.0005   # fixed cost per service step (Section 5 experiment)
     tau: float = 1e-6   # cost per unit of max-driven footprint
@@ -70,6 +71,12 @@ WORKLOADS = {
                 deltas=(256,), online=True,
                 note="Poisson arrivals, mean gap 0.05; prompt LN(ln1024,1) in [16,32768]; "
                      "output LN(ln512,1.3) in [1,16384]"),
+    # Section 5.2: 400 offered requests, o ~ U{1..1000}, price p0 o with p0 = 1/500, and a request in
+    # length bucket b = ceil(o / 100) accepts with probability max{0, 1 - o / ((2b - 1) 100)}; the
+    # accepted requests (in offer order) form the instance, served with B = 50 and no KV cap.
+    6: Workload(6, "profit-experiment", 10_000, 400, 6000, B=(50,), kv_caps=(KV_INF,),
+                deltas=(50, 100, 150, 250, 300, 400, 500), ragged=True,
+                note="400 offered, o ~ U{1..1000}, bucketed acceptance; accepted requests at t=0"),
 }
 
 
@@ -118,18 +125,33 @@ def _draw_chunk(wl: Workload, chunk: int, rows: int, replica: int = 0):
         arrival = _poisson_arrivals(rng, shape, 0.05)
         prompt = _lognormal_int(rng, shape, 1024, 1.0, 16, 32768)
         output = _lognormal_int(rng, shape, 512, 1.3, 1, 16384)
+    elif wl.wid == 6:
+        offered = rng.integers(1, 1001, size=shape)
+        u = rng.random(shape)
+        bucket = (offered + 99) // 100
+        keep = u < np.maximum(0.0, 1.0 - offered / ((2 * bucket - 1) * 100.0))
+        count = keep.sum(axis=1).astype(np.int32)
+        arrival = np.zeros(shape, np.int32)
+        prompt = np.zeros(shape, np.int32)
+        output = np.zeros(shape, np.int32)
+        for r in range(rows):                       # accepted requests first, in offer order
+            acc = offered[r][keep[r]]
+            output[r, :acc.size] = acc
+        return arrival, prompt, output, count
     else:  # pragma: no cover
         raise ValueError(f"unknown workload {wl.wid}")
-    return arrival, prompt, output
+    return arrival, prompt, output, None
 
 
-def generate(wid: int, instances=None, replica: int = 0):
+def generate(wid: int, instances=None, replica: int = 0, with_counts: bool = False):
     """Return (arrival, prompt, output), each int32 of shape (len(instances), n).
 
     ``instances`` is None (all instances), an int m (the first m) or an
     iterable of instance ids.  Instance i is identical whichever way it is
     requested.  ``replica`` r > 0 draws an independent set of the same shape
     (seed sequence [seed, chunk, r]); multi-GPU runs give rank r replica r.
+    ``with_counts`` appends the per-instance request counts (all n except for
+    ragged workloads, whose instance i uses its first counts[i] slots).
     """
     wl = WORKLOADS[wid]
     if instances is None:
@@ -143,6 +165,7 @@ def generate(wid: int, instances=None, replica: int = 0):
     per = chunk_instances(wl.n_per_instance)
     n = wl.n_per_instance
     out = [np.empty((ids.size, n), np.int32) for _ in range(3)]
+    cnt = np.empty(ids.size, np.int32)
     chunks = ids // per
     for c in np.unique(chunks):
         sel = np.nonzero(chunks == c)[0]
@@ -152,6 +175,9 @@ def generate(wid: int, instances=None, replica: int = 0):
         arrs = _draw_chunk(wl, int(c), rows, replica)
         for k in range(3):
             out[k][sel] = arrs[k][ids[sel] % per]
+        cnt[sel] = arrs[3][ids[sel] % per] if arrs[3] is not None else n
+    if with_counts:
+        return tuple(out) + (cnt,)
     return tuple(out)
 
 

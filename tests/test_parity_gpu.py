@@ -39,17 +39,19 @@ def assert_records_equal(g, r, ctx=""):
             np.testing.assert_array_equal(g[f], r[f], err_msg=f"{ctx} {f}")
 
 
-def run_both(S, O, a, p, o, B, policies, deltas, kv, epoch, per_request=True, max_steps=0, check=True):
+def run_both(S, O, a, p, o, B, policies, deltas, kv, epoch, per_request=True, max_steps=0, check=True,
+             counts=None):
     n_inst, n = a.shape
     sm = S.Simulator(n_inst, n, B, max_steps=max_steps, epoch=epoch)
     try:
-        res = sm.sweep(a, p, o, policies, deltas, kv, per_request=per_request)
+        res = sm.sweep(a, p, o, policies, deltas, kv, per_request=per_request, counts=counts)
     finally:
         sm.close()
     assert res["launches"] == 4
     if check:
         for i, (pol, d) in enumerate(zip(policies, deltas)):
-            rec, st, co = O.run(pol, B, d, kv, a, p, o, max_steps=max_steps, per_request=per_request)
+            rec, st, co = O.run(pol, B, d, kv, a, p, o, max_steps=max_steps, per_request=per_request,
+                                counts=counts)
             assert_records_equal(res["records"][i], rec, f"{pol} d={d} epoch={epoch}")
             if per_request:
                 np.testing.assert_array_equal(res["start"][i], st, err_msg=f"start {pol} {d}")
@@ -170,6 +172,35 @@ def test_online_sweep_full_size_sampled(S, O):
             assert s["T_busy"] == int(R[i]["T_busy"].sum()) and s["E"] == int(R[i]["E"].sum())
             assert s["n_ok"] == wl.n_instances and s["status"] == 0
             np.testing.assert_allclose(s["cost"], R[i]["cost"].sum(), rtol=1e-12)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_profit_experiment_workload_ragged(S, O, epoch):
+    """Section 5.2's design: instances of 150-250 accepted requests in 400 slots."""
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o, cnt = W.generate(6, 64, with_counts=True)
+    assert cnt.min() < 400
+    pols = ["fcfs", "ljf"] + ["isjl"] * 7
+    ds = [0, 0, 50, 100, 150, 250, 300, 400, 500]
+    run_both(S, O, a, p, o, 50, pols, ds, INF, epoch, counts=cnt)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_ragged_counts_edges(S, O, epoch):
+    """Empty instances, full instances, and an out-of-range count (INVALID_ARG)."""
+    rng = np.random.default_rng(9)
+    n = 70
+    a = np.sort(rng.integers(0, 90, (6, n)), axis=1).astype(np.int32)
+    p = rng.integers(0, 20, (6, n)).astype(np.int32)
+    o = rng.integers(1, 60, (6, n)).astype(np.int32)
+    cnt = np.array([0, n, 1, 33, 0, 64], np.int32)
+    run_both(S, O, a, p, o, 8, ["fcfs", "ljf", "isjl", "isjl"], [0, 0, 4, INF], 200, epoch, counts=cnt)
+    bad = cnt.copy()
+    bad[2] = n + 1
+    res = run_both(S, O, a, p, o, 8, ["isjl"], [4], 200, epoch, counts=bad, check=False)
+    assert res["records"][0]["status"][2] == 1 and (np.delete(res["records"][0]["status"], 2) == 0).all()
+    rec, _, _ = O.run("isjl", 8, 4, 200, a, p, o, counts=bad)
+    assert_records_equal(res["records"][0], rec)
 
 
 # ---- edge cases -------------------------------------------------------------
