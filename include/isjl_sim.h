@@ -54,9 +54,12 @@ typedef enum {
 } isjl_status;
 
 typedef enum {
-    ISJL_POLICY_FCFS = 0,
-    ISJL_POLICY_LJF = 1,
-    ISJL_POLICY_ISJL = 2
+    ISJL_POLICY_FCFS = 0,       /* arrival order, continuous batching; ignores delta */
+    ISJL_POLICY_LJF = 1,        /* Algorithm 1, static batches of the longest; ignores delta */
+    ISJL_POLICY_ISJL = 2,       /* Algorithm 2 (beta = alpha = delta) */
+    ISJL_POLICY_SJF = 3,        /* shortest first, continuous batching (Section 6 baseline); ignores delta */
+    ISJL_POLICY_ISJL_BETA = 4   /* Algorithm "ISJL": beta = (sqrt(17) - 1) / 4 * delta replaces alpha in the
+                                   packing thresholds (o_1 - o_j + beta); defined by the paper for B = 2 */
 } isjl_policy;
 
 #define ISJL_DELTA_INF 2147483647   /* fairness budget infinity: Eq. 1 is vacuous */
@@ -161,7 +164,7 @@ isjl_status isjl_sim_create(const isjl_config *cfg, isjl_sim **out);
 void isjl_sim_destroy(isjl_sim *sim);
 
 /* Simulate every instance under one policy.  delta: fairness budget >= 0
- * (ISJL_DELTA_INF = none; FCFS and LJF ignore it except for counting
+ * (ISJL_DELTA_INF = none; FCFS, LJF and SJF ignore it except for counting
  * violations).  kv_cap >= 1 (ISJL_KV_INF = none).  Asynchronous on stream:
  * validation of the lengths (INFEASIBLE / INVALID_ARG per instance) happens on
  * the device and is reported by isjl_sim_metrics and the records.

@@ -35,6 +35,8 @@
 #define OR_FCFS 0
 #define OR_LJF  1
 #define OR_ISJL 2
+#define OR_SJF  3   /* shortest first, continuous batching (Section 6 baseline) */
+#define OR_ISJL_BETA 4   /* Algorithm "ISJL" with beta = (sqrt(17) - 1) / 4 * alpha */
 
 #define OR_OK            0
 #define OR_INVALID_ARG   1
@@ -56,7 +58,7 @@ typedef struct {
 
 typedef struct {
     int n, B, policy;
-    int64_t alpha, kv_cap;
+    int64_t alpha, beta, kv_cap;
     const int32_t *arr;
     int32_t *o;
     int32_t *status, *a, *start, *compl;
@@ -108,6 +110,47 @@ static int64_t a_max(const sim_t *s) {
     int64_t m = 0;
     for (int q = 0; q < s->run_cnt; ++q) m = max64(m, s->a[s->run[q]]);
     return m;
+}
+
+/* beta = floor((sqrt(17) - 1) / 4 * alpha), exactly: the largest m >= 0 with
+ * 4m + alpha <= alpha * sqrt(17), i.e. (4m + alpha)^2 <= 17 alpha^2.  Only
+ * floor(beta) matters: o_1 - o_2 + beta is compared with integer sums. */
+static int64_t beta_of(int64_t alpha) {
+    if (alpha > 1000000) return alpha;           /* no plan can exist: o <= 65535 < alpha */
+    int64_t m = (int64_t)(0.780776406404415 * (double)alpha);
+    while (m > 0 && (4 * m + alpha) * (4 * m + alpha) > 17 * alpha * alpha) m--;
+    while ((4 * (m + 1) + alpha) * (4 * (m + 1) + alpha) <= 17 * alpha * alpha) m++;
+    return m;
+}
+
+/* shortest released request that is neither running, done nor planned */
+static int32_t shortest_waiting(const sim_t *s, int64_t k) {
+    for (int p = s->n - 1; p >= 0; --p) {
+        int32_t i = s->by_len[p];
+        if (s->status[i] == ST_WAIT && s->arr[i] <= k) {
+            /* among equal lengths the lower index goes first */
+            int32_t best = i;
+            for (int q = p - 1; q >= 0 && s->o[s->by_len[q]] == s->o[i]; --q) {
+                int32_t j = s->by_len[q];
+                if (s->status[j] == ST_WAIT && s->arr[j] <= k) best = j;
+            }
+            return best;
+        }
+    }
+    return -1;
+}
+
+/* ---- SJF (Section 2.1 example, continuous-batching remark; Section 6) ----- */
+/* Each step admit released requests shortest first (ties: lower index) while
+ * a slot is free and the KV reservation fits; the first that does not fit
+ * ends admissions.  No fairness gate. */
+static void sjf_admit(sim_t *s, int64_t k) {
+    while (s->run_cnt < s->B) {
+        int32_t i = shortest_waiting(s, k);
+        if (i < 0) break;
+        if (s->kv_sum + s->o[i] > s->kv_cap) break;
+        start_job(s, i, k, 0);
+    }
 }
 
 /* ---- FCFS (Section 2.1 example, continuous-batching remark) -------------- */
@@ -169,12 +212,13 @@ static int isjl_phase_one(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int
     for (int p = 0; p < q; ++p) if ((int64_t)s->o[Q[p]] > al) cnt_long++;
     int n_long = cnt_long < s->B ? cnt_long : s->B;
     const int64_t o1 = s->o[Q[0]];
-    const int64_t theta = min64(2 * al, o1 - (int64_t)s->o[Q[n_long - 1]] + al);
+    const int64_t be = s->beta;   /* beta = alpha (Algorithm 2), or Algorithm "ISJL"'s beta */
+    const int64_t theta = min64(2 * al, o1 - (int64_t)s->o[Q[n_long - 1]] + be);
 
-    /* packing budgets: workers 2..M get cap_j = min{2 alpha, o_1 - o_j + alpha},
+    /* packing budgets: workers 2..M get cap_j = min{2 alpha, o_1 - o_j + beta},
      * workers M+1..B get alpha */
     for (int j = 1; j <= s->B; ++j) { packsum[j] = 0; budget[j] = -1; }
-    for (int j = 2; j <= n_long; ++j) budget[j] = min64(2 * al, o1 - (int64_t)s->o[Q[j - 1]] + al);
+    for (int j = 2; j <= n_long; ++j) budget[j] = min64(2 * al, o1 - (int64_t)s->o[Q[j - 1]] + be);
     for (int j = n_long + 1; j <= s->B; ++j) budget[j] = al;
 
     /* the long requests leave the queue (worker j will run o_j) */
@@ -267,7 +311,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
                int32_t *start_out, int32_t *compl_out, or_record *rec)
 {
     memset(rec, 0, sizeof(*rec));
-    if (n < 0 || B < 1 || delta < 0 || kv_cap < 1 || policy < 0 || policy > 2 || (n > 0 && (!arrival || !prompt || !output))) {
+    if (n < 0 || B < 1 || delta < 0 || kv_cap < 1 || policy < 0 || policy > 4 || (n > 0 && (!arrival || !prompt || !output))) {
         rec->status = OR_INVALID_ARG; return OR_INVALID_ARG;
     }
     if (n == 0) return OR_OK;   /* an empty instance: nothing runs, every counter is 0 */
@@ -278,7 +322,10 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     }
     sim_t S; memset(&S, 0, sizeof(S));
     sim_t *s = &S;
-    s->n = n; s->B = B; s->policy = policy; s->alpha = delta; s->kv_cap = kv_cap; s->arr = arrival;
+    s->n = n; s->B = B; s->policy = policy == OR_ISJL_BETA ? OR_ISJL : policy; s->alpha = delta;
+    s->beta = policy == OR_ISJL_BETA ? beta_of(delta) : delta;
+    s->kv_cap = kv_cap; s->arr = arrival;
+    policy = s->policy;
     s->o = malloc(sizeof(int32_t) * n);
     s->status = malloc(sizeof(int32_t) * n);
     s->a = malloc(sizeof(int32_t) * n);
@@ -348,6 +395,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
         /* admission */
         if (policy == OR_FCFS) fcfs_admit(s, k);
         else if (policy == OR_LJF) ljf_admit(s, k);
+        else if (policy == OR_SJF) sjf_admit(s, k);
         else isjl_admit(s, k, Q, packsum, budget);
 
         /* serve step k: every running request processes token r_i = a_i + 1 */
@@ -420,3 +468,4 @@ int oracle_run_batch(int policy, int B, int64_t delta, int64_t kv_cap, int n_ins
 }
 
 int oracle_record_size(void) { return (int)sizeof(or_record); }
+int64_t oracle_beta(int64_t alpha) { return beta_of(alpha); }

@@ -20,7 +20,7 @@ import numpy as np
 from . import build as _build
 
 INT32_MAX = 2**31 - 1
-POLICIES = {"fcfs": 0, "ljf": 1, "isjl": 2}
+POLICIES = {"fcfs": 0, "ljf": 1, "isjl": 2, "sjf": 3, "isjl_beta": 4}
 STATUS = {0: "ok", 1: "invalid_arg", 2: "infeasible", 3: "oom", 5: "step_limit"}
 
 RECORD_FIELDS_I64 = ["T_make", "T_busy", "O", "Q", "W", "E", "token_adv",
@@ -45,6 +45,8 @@ def lib():
                                        ctypes.c_int64, p32, p32, ctypes.c_void_p]
         L.oracle_run_batch.restype = ctypes.c_int
         L.oracle_record_size.restype = ctypes.c_int
+        L.oracle_beta.argtypes = [ctypes.c_int64]
+        L.oracle_beta.restype = ctypes.c_int64
         L.oracle_opt_makespan.argtypes = [ctypes.c_int, p32, p32, ctypes.c_int, ctypes.c_int64,
                                           ctypes.c_int64, ctypes.c_int64]
         L.oracle_opt_makespan.restype = ctypes.c_int64
@@ -114,6 +116,11 @@ def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p
         st = st[0] if per_request else None
         co = co[0] if per_request else None
     return rec, st, co
+
+
+def beta(alpha):
+    """floor((sqrt(17) - 1) / 4 * alpha), Algorithm "ISJL"'s beta, exact."""
+    return int(lib().oracle_beta(int(alpha)))
 
 
 def opt_makespan(arrival, o, B, delta, kv_cap=INT32_MAX, max_T=100_000):

@@ -52,7 +52,7 @@ void free_all(isjl_sim *s) {
 bool valid_runs(int32_t n_runs, const int32_t *policies, const int32_t *deltas) {
     if (n_runs < 1 || n_runs > ISJL_MAX_RUNS || !policies || !deltas) return false;
     for (int i = 0; i < n_runs; ++i) {
-        if (policies[i] < ISJL_POLICY_FCFS || policies[i] > ISJL_POLICY_ISJL) return false;
+        if (policies[i] < ISJL_POLICY_FCFS || policies[i] > ISJL_POLICY_ISJL_BETA) return false;
         if (deltas[i] < 0) return false;
     }
     return true;
@@ -133,7 +133,11 @@ isjl_status isjl_sim_run_sweep(isjl_sim *s, int32_t n_runs, const int32_t *polic
     auto mark = [&](int i) { return !timing || cudaEventRecord(s->ev[i], st) == cudaSuccess; };
     RunList runs;
     std::memset(&runs, 0, sizeof(runs));
-    for (int i = 0; i < n_runs; ++i) { runs.policy[i] = policies[i]; runs.delta[i] = deltas[i]; }
+    for (int i = 0; i < n_runs; ++i) {
+        runs.policy[i] = policies[i];
+        runs.delta[i] = deltas[i];
+        runs.beta[i] = isjl::run_beta(policies[i], deltas[i]);
+    }
 
     if (cudaMemsetAsync(s->d_counter, 0, sizeof(int32_t), st) != cudaSuccess ||
         cudaMemsetAsync(s->d_status, 0, sizeof(int32_t), st) != cudaSuccess || !mark(0))

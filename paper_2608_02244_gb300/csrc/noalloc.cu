@@ -66,7 +66,7 @@ extern "C" isjl_status isjl_sim_run_sweep_noalloc(const isjl_config *cfg, int32_
         return ISJL_ERR_INVALID_ARG;
     if (n_runs < 1 || n_runs > ISJL_MAX_RUNS || !policies || !deltas) return ISJL_ERR_INVALID_ARG;
     for (int i = 0; i < n_runs; ++i)
-        if (policies[i] < ISJL_POLICY_FCFS || policies[i] > ISJL_POLICY_ISJL || deltas[i] < 0)
+        if (policies[i] < ISJL_POLICY_FCFS || policies[i] > ISJL_POLICY_ISJL_BETA || deltas[i] < 0)
             return ISJL_ERR_INVALID_ARG;
 
     // workspace layout inside the fixed array
@@ -136,7 +136,11 @@ extern "C" isjl_status isjl_sim_run_sweep_noalloc(const isjl_config *cfg, int32_
     a.c = cfg->c;
     a.tau = cfg->tau;
     a.p0 = cfg->p0;
-    for (int i = 0; i < n_runs; ++i) { a.runs.policy[i] = policies[i]; a.runs.delta[i] = deltas[i]; }
+    for (int i = 0; i < n_runs; ++i) {
+        a.runs.policy[i] = policies[i];
+        a.runs.delta[i] = deltas[i];
+        a.runs.beta[i] = isjl::run_beta(policies[i], deltas[i]);
+    }
     if (isjl::launch_sim(a, epoch, warps, st) != cudaSuccess) return ISJL_ERR_CUDA;
     return ISJL_OK;
 }

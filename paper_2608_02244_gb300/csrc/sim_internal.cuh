@@ -30,7 +30,21 @@ struct InstStats {
 struct RunList {
     int32_t policy[ISJL_MAX_RUNS];
     int32_t delta[ISJL_MAX_RUNS];
+    int32_t beta[ISJL_MAX_RUNS];    // ISJL packing slack: delta, or Algorithm "ISJL"'s beta
 };
+
+// floor((sqrt(17) - 1) / 4 * alpha) exactly: the largest m with (4m + alpha)^2 <= 17 alpha^2
+inline int32_t isjl_beta(int32_t alpha) {
+    if (alpha > 1000000) return alpha;   // no plan exists when alpha >= every length
+    const int64_t a = alpha;
+    int64_t m = (int64_t)(0.780776406404415 * (double)alpha);
+    while (m > 0 && (4 * m + a) * (4 * m + a) > 17 * a * a) m--;
+    while ((4 * (m + 1) + a) * (4 * (m + 1) + a) <= 17 * a * a) m++;
+    return (int32_t)m;
+}
+inline int32_t run_beta(int32_t policy, int32_t delta) {
+    return policy == ISJL_POLICY_ISJL_BETA ? isjl_beta(delta) : delta;
+}
 
 struct SimArgs {
     const int32_t *arrival;    // [N] instance-major

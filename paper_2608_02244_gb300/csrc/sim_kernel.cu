@@ -120,6 +120,22 @@ __device__ __forceinline__ void bs_clear(const WarpSmem &S, int p, int lane) {
     __syncwarp();
 }
 
+// highest pending sorted position, -1 if none (uniform call)
+__device__ __forceinline__ int bs_last(const WarpSmem &S, int words1, int lane) {
+    for (int b1 = (words1 - 1) & ~31; b1 >= 0; b1 -= 32) {
+        const int idx = b1 + lane;
+        const uint32_t x = idx < words1 ? S.pend1[idx] : 0u;
+        const unsigned b = __ballot_sync(kFull, x != 0u);
+        if (b) {
+            const int l = 31 - __clz(b);
+            const uint32_t xx = __shfl_sync(kFull, x, l);
+            const int ww = ((b1 + l) << 5) + 31 - __clz(xx);
+            return (ww << 5) + 31 - __clz(S.pend0[ww]);
+        }
+    }
+    return -1;
+}
+
 // number of pending positions < P (uniform call)
 __device__ __forceinline__ int bs_count_below(const WarpSmem &S, int words0, int P, int lane) {
     const int full = P >> 5;
@@ -148,8 +164,11 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     const int64_t base = inst * (int64_t)n_slots;
     const InstStats is = A.inst[inst];
     const int n = is.n;                             // requests of this instance (<= n_slots)
-    const int policy = A.runs.policy[run];
+    const int policy_in = A.runs.policy[run];
+    // Algorithm "ISJL" runs the ISJL machinery with beta in the packing thresholds
+    const int policy = policy_in == ISJL_POLICY_ISJL_BETA ? ISJL_POLICY_ISJL : policy_in;
     const int64_t alpha = A.runs.delta[run];
+    const int64_t beta = A.runs.beta[run];
     const int64_t kv_cap = A.kv_cap;
     const int32_t *__restrict__ arr = A.arrival + base;
     const int32_t *__restrict__ oarr = A.o + base;
@@ -340,6 +359,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (p1 >= n) { broken = true; return; }
             const int64_t o1 = osrt[p1];
             const int p2 = bs_next(S, words0, words1, p1 + 1, lane);
+            // cap_j = min{2 alpha, o_1 - o_j + beta}, theta likewise (beta = alpha in Algorithm 2)
             if (p2 >= n) { broken = true; return; }
             if ((int64_t)osrt[p2] <= alpha) return;             // o_2 <= alpha: Phase TWO
             // M = min{B, #{o > alpha}} over Q(k)
@@ -364,7 +384,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     L1 = e;
                     if (lane == 0) { S.shead[0] = e; S.stail[0] = e; pnext[e] = kNone; }
                 } else {
-                    const int64_t cap = min(2 * alpha, o1 - oe + alpha);
+                    const int64_t cap = min(2 * alpha, o1 - oe + beta);
                     if (lane == 0) S.slong[j] = e;
                     if (lane == 0) S.srem[j] = (int32_t)cap;
                 }
@@ -372,7 +392,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             }
             __syncwarp();
             pend -= nl;
-            const int64_t theta = min(2 * alpha, o1 - o_last + alpha);
+            const int64_t theta = min(2 * alpha, o1 - o_last + beta);
             // first fit of the shorter requests, in sorted order
             int maxrem = -1;
             for (int w = lane; w < B; w += 32) maxrem = max(maxrem, S.srem[w]);
@@ -456,6 +476,22 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     start(fcfs, fo, w);
                     fcfs++;
                     fo = -1;
+                }
+            } else if (policy == ISJL_POLICY_SJF) {
+                // shortest released request first (ties: lower index), continuous batching
+                while (run_cnt < B && pend > 0) {
+                    const int hi = bs_last(S, words1, lane);
+                    if (hi < 0 || hi >= n) { broken = true; return; }
+                    const int omin = osrt[hi];
+                    const int p = bs_next(S, words0, words1, first_pos_le(osrt, n, omin), lane);
+                    if (p >= n) { broken = true; return; }
+                    if (kv_sum + omin > kv_cap) break;
+                    const int w = lowest_worker(vmask & ~busy, lane);
+                    if (w < 0) { broken = true; return; }
+                    const int e = perm[p];
+                    bs_clear(S, p, lane);
+                    pend--;
+                    start(e, omin, w);
                 }
             } else if (policy == ISJL_POLICY_LJF) {
                 // static batch of the longest released requests when nothing runs

@@ -50,3 +50,21 @@ def test_b3_misses_match_recorded_findings(computed):
         assert fg == rec[(3, d, "gamma")]
     # the bound holds at both ends of the budget range
     assert computed[(3, 0)] == ([], []) and computed[(3, INF)] == ([], [])
+
+
+def test_b2_isjl_with_optimal_beta_meets_its_bound():
+    """Theorem "Competitive ratio of Algorithm ISJL" (B = 2): with
+    beta = (sqrt(17) - 1)/4 alpha, T_OPT / T >= min{(a + 2b)/(a + 3b), 4a/(6a - b)}
+    (about 0.766), on every tiny instance, offline without a KV cap."""
+    import math
+    from oracle import oracle as O
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, out = W.generate(2)
+    o = p + out
+    for d in (1, 2, 4, 8):
+        beta = (math.sqrt(17) - 1) / 4 * d
+        bound = min((d + 2 * beta) / (d + 3 * beta), 4 * d / (6 * d - beta))
+        rec, _, _ = O.run("isjl_beta", 2, d, INF, a, p, out, per_request=False)
+        assert (rec["violations"] == 0).all()
+        for i in range(len(o)):
+            assert O.opt_makespan(a[i], o[i], 2, d) >= bound * rec["T_make"][i] - 1e-9, (d, i)

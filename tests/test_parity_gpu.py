@@ -75,8 +75,8 @@ def test_single_instance_workload(S, O, epoch):
 def test_tiny_exhaustive_workload(S, O, epoch, B, kv):
     from paper_2608_02244_gb300 import workloads as W
     a, p, o = W.generate(2)
-    pols = ["isjl"] * 5 + ["fcfs", "ljf"]
-    ds = [0, 1, 2, 4, INF, 0, 0]
+    pols = ["isjl"] * 5 + ["fcfs", "ljf", "sjf"] + ["isjl_beta"] * 3
+    ds = [0, 1, 2, 4, INF, 0, 0, 0, 1, 2, 4]
     run_both(S, O, a, p, o, B, pols, ds, kv, epoch)
 
 
@@ -119,8 +119,8 @@ def test_online_sweep_workload_subset(S, O, epoch):
     """16 full-size instances (n = 1000, ragged against 32) of the online sweep."""
     from paper_2608_02244_gb300 import workloads as W
     a, p, o = W.generate(3, 16)
-    pols = ["fcfs", "ljf"] + ["isjl"] * 5
-    ds = [0, 0, 16, 64, 256, 1024, INF]
+    pols = ["fcfs", "ljf"] + ["isjl"] * 5 + ["sjf", "isjl_beta", "isjl_beta"]
+    ds = [0, 0, 16, 64, 256, 1024, INF, 0, 64, 1024]
     run_both(S, O, a, p, o, 256, pols, ds, 200_000, epoch)
 
 
@@ -128,8 +128,8 @@ def test_online_sweep_workload_subset(S, O, epoch):
 def test_heavy_tail_workload_subset(S, O, epoch):
     from paper_2608_02244_gb300 import workloads as W
     a, p, o = W.generate(4, 48)
-    pols = ["fcfs", "ljf", "isjl", "isjl", "isjl"]
-    ds = [0, 0, 32, 128, 512]
+    pols = ["fcfs", "ljf", "isjl", "isjl", "isjl", "sjf", "isjl_beta"]
+    ds = [0, 0, 32, 128, 512, 0, 128]
     run_both(S, O, a, p, o, 128, pols, ds, 65_536, epoch)
 
 
@@ -180,8 +180,8 @@ def test_profit_experiment_workload_ragged(S, O, epoch):
     from paper_2608_02244_gb300 import workloads as W
     a, p, o, cnt = W.generate(6, 64, with_counts=True)
     assert cnt.min() < 400
-    pols = ["fcfs", "ljf"] + ["isjl"] * 7
-    ds = [0, 0, 50, 100, 150, 250, 300, 400, 500]
+    pols = ["fcfs", "ljf"] + ["isjl"] * 7 + ["sjf", "isjl_beta"]
+    ds = [0, 0, 50, 100, 150, 250, 300, 400, 500, 0, 150]
     run_both(S, O, a, p, o, 50, pols, ds, INF, epoch, counts=cnt)
 
 
@@ -194,7 +194,8 @@ def test_ragged_counts_edges(S, O, epoch):
     p = rng.integers(0, 20, (6, n)).astype(np.int32)
     o = rng.integers(1, 60, (6, n)).astype(np.int32)
     cnt = np.array([0, n, 1, 33, 0, 64], np.int32)
-    run_both(S, O, a, p, o, 8, ["fcfs", "ljf", "isjl", "isjl"], [0, 0, 4, INF], 200, epoch, counts=cnt)
+    run_both(S, O, a, p, o, 8, ["fcfs", "ljf", "isjl", "isjl", "sjf", "isjl_beta"], [0, 0, 4, INF, 0, 4], 200, epoch,
+             counts=cnt)
     bad = cnt.copy()
     bad[2] = n + 1
     res = run_both(S, O, a, p, o, 8, ["isjl"], [4], 200, epoch, counts=bad, check=False)
@@ -223,8 +224,9 @@ def test_edge_shapes(S, O, epoch):
         cases.append((a, p, o, B))
     for a, p, o, B in cases:
         kv = int((p + o).max()) + 50
-        run_both(S, O, a, p, o, B, ["fcfs", "ljf", "isjl", "isjl", "isjl"], [0, 0, 0, 5, INF], kv, epoch)
-        run_both(S, O, a, p, o, B, ["isjl", "isjl"], [3, 40], INF, epoch)
+        run_both(S, O, a, p, o, B, ["fcfs", "ljf", "isjl", "isjl", "isjl", "sjf", "isjl_beta"],
+                 [0, 0, 0, 5, INF, 0, 5], kv, epoch)
+        run_both(S, O, a, p, o, B, ["isjl", "isjl", "sjf", "isjl_beta"], [3, 40, 0, 40], INF, epoch)
 
 
 @pytest.mark.parametrize("epoch", EPOCHS)
@@ -235,7 +237,8 @@ def test_radix_path_small_count(S, O, epoch):
     a = np.sort(rng.integers(0, 30000, (2, n)), axis=1).astype(np.int32)
     p = rng.integers(0, 200, (2, n)).astype(np.int32)
     o = rng.integers(1, 300, (2, n)).astype(np.int32)
-    run_both(S, O, a, p, o, 40, ["fcfs", "ljf", "isjl", "isjl"], [0, 0, 60, INF], 3000, epoch)
+    run_both(S, O, a, p, o, 40, ["fcfs", "ljf", "isjl", "isjl", "sjf", "isjl_beta"], [0, 0, 60, INF, 0, 60], 3000,
+             epoch)
 
 
 @pytest.mark.parametrize("epoch", EPOCHS)
