@@ -94,6 +94,11 @@ typedef struct {
                                 count[i] slots (0..n_per_instance; 0 = an empty instance, all
                                 counters 0); NULL = every instance uses all n_per_instance.  A
                                 count outside 0..n_per_instance makes that instance INVALID_ARG. */
+    const int32_t *slack;    /* device, same shape as arrival, or NULL: upper-bound slack
+                                e_i = u_i - o_i >= 0 of length predictions (Robust-ISJL, Section
+                                3.3).  Every policy then plans with u_i = o_i + e_i (order, packing,
+                                KV reservation) while request i still finishes after o_i tokens and
+                                the fairness gate uses true progress.  NULL = exact lengths. */
 } isjl_instances;
 
 /* One result record per (run, instance).  Integers are exact; the doubles

@@ -27,6 +27,10 @@
  *   - A request started in step k runs in step k; completion c_i = (last step
  *     it ran) + 1; T_busy counts nonempty steps, T_make = max c_i.
  *   - ISJL: see isjl_admit() below.
+ *   - Robust-ISJL (Section 3.3): with an upper-bound slack e_i >= 0 the
+ *     policies plan with u_i = o_i + e_i (sorting, M, cap_j, packs, Phase TWO
+ *     order, KV reservation of u_i); requests still finish after o_i tokens
+ *     and the gate uses their true progress.  e = 0 is the clairvoyant case.
  */
 #include <stdint.h>
 #include <stdlib.h>
@@ -60,7 +64,8 @@ typedef struct {
     int n, B, policy;
     int64_t alpha, beta, kv_cap;
     const int32_t *arr;
-    int32_t *o;
+    int32_t *o;               /* planning length u_i (= o_i without predictions) */
+    int32_t *ot;              /* true length o_i */
     int32_t *status, *a, *start, *compl;
     int32_t *by_len;          /* job ids sorted by (o desc, idx asc) */
     /* running set */
@@ -306,7 +311,7 @@ static void isjl_admit(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_
  * (INT32_MAX = no constraint; ignored by FCFS and LJF except for counting
  * violations).  start_out/compl_out may be NULL.  Returns the status. */
 int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
-               const int32_t *arrival, const int32_t *prompt, const int32_t *output,
+               const int32_t *arrival, const int32_t *prompt, const int32_t *output, const int32_t *slack,
                double c, double tau, double p0, int64_t max_steps,
                int32_t *start_out, int32_t *compl_out, or_record *rec)
 {
@@ -316,7 +321,8 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     }
     if (n == 0) return OR_OK;   /* an empty instance: nothing runs, every counter is 0 */
     for (int i = 0; i < n; ++i) {
-        if (arrival[i] < 0 || prompt[i] < 0 || output[i] < 0 || (i > 0 && arrival[i] < arrival[i - 1])) {
+        if (arrival[i] < 0 || prompt[i] < 0 || output[i] < 0 || (slack && slack[i] < 0) ||
+            (i > 0 && arrival[i] < arrival[i - 1])) {
             rec->status = OR_INVALID_ARG; return OR_INVALID_ARG;
         }
     }
@@ -327,6 +333,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     s->kv_cap = kv_cap; s->arr = arrival;
     policy = s->policy;
     s->o = malloc(sizeof(int32_t) * n);
+    s->ot = malloc(sizeof(int32_t) * n);
     s->status = malloc(sizeof(int32_t) * n);
     s->a = malloc(sizeof(int32_t) * n);
     s->start = malloc(sizeof(int32_t) * n);
@@ -343,7 +350,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     s->job_worker = malloc(sizeof(int32_t) * n);
     s->long_of = malloc(sizeof(int32_t) * (size_t)(B + 1));
     int status = OR_OK;
-    if (!s->o || !s->status || !s->a || !s->start || !s->compl || !s->by_len || !s->run || !Q ||
+    if (!s->o || !s->ot || !s->status || !s->a || !s->start || !s->compl || !s->by_len || !s->run || !Q ||
         !packsum || !budget || !s->worker_job || !s->plan_head || !s->plan_tail || !s->plan_next || !s->job_worker || !s->long_of) {
         status = OR_OOM; goto done;
     }
@@ -352,8 +359,10 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     int64_t O = 0, Qsum = 0, sumA = 0, maxA = 0;
     for (int i = 0; i < n; ++i) {
         int64_t oi = (int64_t)prompt[i] + output[i];
-        if (oi < 1 || oi > kv_cap || oi > INT32_MAX / 2) { status = OR_INFEASIBLE; goto done; }
-        s->o[i] = (int32_t)oi;
+        int64_t ui = oi + (slack ? slack[i] : 0);           /* planning length u_i >= o_i */
+        if (oi < 1 || ui > kv_cap || ui > INT32_MAX / 2) { status = OR_INFEASIBLE; goto done; }
+        s->o[i] = (int32_t)ui;
+        s->ot[i] = (int32_t)oi;
         O += oi;
         Qsum += oi * (oi + 1) / 2;          /* Eq. intrinsic-resource-cost */
         sumA += arrival[i];
@@ -377,7 +386,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
         int w = 0;
         for (int q = 0; q < s->run_cnt; ++q) {
             int32_t i = s->run[q];
-            if (s->a[i] == s->o[i]) {
+            if (s->a[i] == s->ot[i]) {
                 s->status[i] = ST_DONE;
                 s->compl[i] = (int32_t)k;
                 s->kv_sum -= s->o[i];
@@ -442,7 +451,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     if (compl_out) memcpy(compl_out, s->compl, sizeof(int32_t) * n);
 done:
     rec->status = status;
-    free(s->o); free(s->status); free(s->a); free(s->start); free(s->compl); free(s->by_len);
+    free(s->o); free(s->ot); free(s->status); free(s->a); free(s->start); free(s->compl); free(s->by_len);
     free(s->run); free(Q); free(packsum); free(budget); free(s->worker_job); free(s->plan_head);
     free(s->plan_tail); free(s->plan_next); free(s->job_worker); free(s->long_of);
     return status;
@@ -452,7 +461,7 @@ done:
  * rec has n_inst entries; start_out/compl_out are n_inst*n or NULL.
  * Returns the first nonzero status, else 0. */
 int oracle_run_batch(int policy, int B, int64_t delta, int64_t kv_cap, int n_inst, int n,
-                     const int32_t *arrival, const int32_t *prompt, const int32_t *output,
+                     const int32_t *arrival, const int32_t *prompt, const int32_t *output, const int32_t *slack,
                      double c, double tau, double p0, int64_t max_steps,
                      int32_t *start_out, int32_t *compl_out, or_record *rec)
 {
@@ -460,7 +469,7 @@ int oracle_run_batch(int policy, int B, int64_t delta, int64_t kv_cap, int n_ins
     for (int t = 0; t < n_inst; ++t) {
         size_t off = (size_t)t * (size_t)n;
         int st = oracle_run(policy, B, delta, kv_cap, n, arrival + off, prompt + off, output + off,
-                            c, tau, p0, max_steps, start_out ? start_out + off : NULL,
+                            slack ? slack + off : NULL, c, tau, p0, max_steps, start_out ? start_out + off : NULL,
                             compl_out ? compl_out + off : NULL, rec + t);
         if (st && !first) first = st;
     }

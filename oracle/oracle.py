@@ -40,7 +40,7 @@ def lib():
         L = ctypes.CDLL(path)
         p32 = ctypes.POINTER(ctypes.c_int32)
         L.oracle_run_batch.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
-                                       ctypes.c_int, ctypes.c_int, p32, p32, p32,
+                                       ctypes.c_int, ctypes.c_int, p32, p32, p32, p32,
                                        ctypes.c_double, ctypes.c_double, ctypes.c_double,
                                        ctypes.c_int64, p32, p32, ctypes.c_void_p]
         L.oracle_run_batch.restype = ctypes.c_int
@@ -65,17 +65,20 @@ def _ptr(a):
 
 
 def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p0=0.002,
-        max_steps=0, per_request=True, counts=None):
+        max_steps=0, per_request=True, counts=None, slack=None):
     """Simulate every instance (row) under one policy and budget.
 
     Returns (records, start, completion); records is a structured array with
     one entry per instance (fields RECORD_DTYPE), start/completion are int32
     arrays shaped like ``arrival`` (None when per_request is False).
     ``counts`` (optional, one per row) limits instance i to its first
-    counts[i] requests (ragged batches); the rest stay -1.
+    counts[i] requests (ragged batches); the rest stay -1.  ``slack`` (optional,
+    shaped like ``arrival``) is the upper-bound slack e_i = u_i - o_i: policies
+    plan with u_i and requests finish after o_i tokens (Robust-ISJL).
     """
     if counts is not None:
         a, p, o = (np.atleast_2d(_i32(x)) for x in (arrival, prompt, output))
+        e = np.atleast_2d(_i32(slack)) if slack is not None else None
         recs, sts, cos = [], [], []
         for i, m in enumerate(np.asarray(counts)):
             m = int(m)
@@ -88,7 +91,7 @@ def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p
                     cos.append(np.full((1, a.shape[1]), -1, np.int32))
                 continue
             r, st, co = run(policy, B, delta, kv_cap, a[i:i + 1, :m], p[i:i + 1, :m], o[i:i + 1, :m], c, tau, p0,
-                            max_steps, per_request)
+                            max_steps, per_request, slack=e[i:i + 1, :m] if e is not None else None)
             recs.append(r)
             if per_request:
                 row = np.full((1, a.shape[1]), -1, np.int32)
@@ -100,15 +103,18 @@ def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p
         rec = np.concatenate(recs)
         return rec, (np.concatenate(sts) if per_request else None), (np.concatenate(cos) if per_request else None)
     a, p, o = _i32(arrival), _i32(prompt), _i32(output)
+    e = _i32(slack) if slack is not None else None
     squeeze = a.ndim == 1
     if squeeze:
         a, p, o = a[None], p[None], o[None]
+        e = e[None] if e is not None else None
     n_inst, n = a.shape
     rec = np.zeros(n_inst, RECORD_DTYPE)
     st = np.full((n_inst, n), -1, np.int32) if per_request else None
     co = np.full((n_inst, n), -1, np.int32) if per_request else None
     lib().oracle_run_batch(POLICIES[policy], int(B), int(delta), int(kv_cap), n_inst, n,
-                           _ptr(a), _ptr(p), _ptr(o), float(c), float(tau), float(p0), int(max_steps),
+                           _ptr(a), _ptr(p), _ptr(o), _ptr(e) if e is not None else None,
+                           float(c), float(tau), float(p0), int(max_steps),
                            _ptr(st) if per_request else None, _ptr(co) if per_request else None,
                            rec.ctypes.data)
     if squeeze:

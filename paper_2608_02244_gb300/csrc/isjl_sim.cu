@@ -15,6 +15,7 @@ struct isjl_sim {
     int device = 0;
     int64_t N = 0;                   // n_instances * n_per_instance
     int32_t *d_o = nullptr, *d_perm = nullptr, *d_osorted = nullptr, *d_posof = nullptr, *d_tmp = nullptr;
+    int32_t *d_otrue = nullptr;      // true lengths, allocated on the first call with slack
     InstStats *d_inst = nullptr;
     int32_t *d_plan_next = nullptr;
     int total_warps = 0;
@@ -43,7 +44,7 @@ cudaError_t dalloc(T **p, size_t count) {
 void free_all(isjl_sim *s) {
     for (cudaEvent_t &e : s->ev)
         if (e) { cudaEventDestroy(e); e = nullptr; }
-    void *ptrs[] = {s->d_o, s->d_perm, s->d_osorted, s->d_posof, s->d_tmp, s->d_inst, s->d_plan_next,
+    void *ptrs[] = {s->d_o, s->d_otrue, s->d_perm, s->d_osorted, s->d_posof, s->d_tmp, s->d_inst, s->d_plan_next,
                     s->d_counter, s->d_status, s->d_summary, s->d_in[0], s->d_in[1], s->d_in[2], s->d_rec_io};
     for (void *p : ptrs)
         if (p) cudaFree(p);
@@ -142,8 +143,14 @@ isjl_status isjl_sim_run_sweep(isjl_sim *s, int32_t n_runs, const int32_t *polic
     if (cudaMemsetAsync(s->d_counter, 0, sizeof(int32_t), st) != cudaSuccess ||
         cudaMemsetAsync(s->d_status, 0, sizeof(int32_t), st) != cudaSuccess || !mark(0))
         return ISJL_ERR_CUDA;
-    if (isjl::launch_derive(in->arrival, in->prompt, in->output, in->count, s->d_o, s->d_inst, c.n_instances,
-                            c.n_per_instance, st) != cudaSuccess || !mark(1))
+    if (in->slack && !s->d_otrue && dalloc(&s->d_otrue, s->N) != cudaSuccess) {
+        cudaGetLastError();
+        s->d_otrue = nullptr;
+        return ISJL_ERR_OOM;
+    }
+    int32_t *otrue = in->slack ? s->d_otrue : nullptr;
+    if (isjl::launch_derive(in->arrival, in->prompt, in->output, in->count, in->slack, s->d_o, otrue, s->d_inst,
+                            c.n_instances, c.n_per_instance, st) != cudaSuccess || !mark(1))
         return ISJL_ERR_CUDA;
     s->last_launches++;
     if (isjl::launch_sort(s->d_o, s->d_inst, s->d_perm, s->d_osorted, s->d_posof, s->d_tmp, c.n_instances,
@@ -155,6 +162,7 @@ isjl_status isjl_sim_run_sweep(isjl_sim *s, int32_t n_runs, const int32_t *polic
     std::memset(&a, 0, sizeof(a));
     a.arrival = in->arrival;
     a.o = s->d_o;
+    a.otrue = otrue;
     a.perm = s->d_perm;
     a.osorted = s->d_osorted;
     a.posof = s->d_posof;

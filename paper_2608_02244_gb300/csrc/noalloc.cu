@@ -79,6 +79,7 @@ extern "C" isjl_status isjl_sim_run_sweep_noalloc(const isjl_config *cfg, int32_
     const size_t os_off = off;       off = align256(off + sizeof(int32_t) * N);
     const size_t pos_off = off;      off = align256(off + sizeof(int32_t) * N);
     const size_t tmp_off = off;      if (big) off = align256(off + sizeof(int32_t) * N);
+    const size_t ot_off = off;       if (in->slack) off = align256(off + sizeof(int32_t) * N);
     const size_t inst_off = off;     off = align256(off + sizeof(isjl::InstStats) * cfg->n_instances);
     const size_t ctr_off = off;      off = align256(off + 2 * sizeof(int32_t));
     const size_t plan_off = off;
@@ -99,14 +100,15 @@ extern "C" isjl_status isjl_sim_run_sweep_noalloc(const isjl_config *cfg, int32_
     int32_t *d_os = reinterpret_cast<int32_t *>(base + os_off);
     int32_t *d_pos = reinterpret_cast<int32_t *>(base + pos_off);
     int32_t *d_tmp = big ? reinterpret_cast<int32_t *>(base + tmp_off) : nullptr;
+    int32_t *d_ot = in->slack ? reinterpret_cast<int32_t *>(base + ot_off) : nullptr;
     isjl::InstStats *d_inst = reinterpret_cast<isjl::InstStats *>(base + inst_off);
     int32_t *d_ctr = reinterpret_cast<int32_t *>(base + ctr_off);
     int32_t *d_plan = reinterpret_cast<int32_t *>(base + plan_off);
 
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (cudaMemsetAsync(d_ctr, 0, 2 * sizeof(int32_t), st) != cudaSuccess) return ISJL_ERR_CUDA;
-    if (isjl::launch_derive(in->arrival, in->prompt, in->output, in->count, d_o, d_inst, cfg->n_instances, n, st) !=
-        cudaSuccess)
+    if (isjl::launch_derive(in->arrival, in->prompt, in->output, in->count, in->slack, d_o, d_ot, d_inst,
+                            cfg->n_instances, n, st) != cudaSuccess)
         return ISJL_ERR_CUDA;
     if (isjl::launch_sort(d_o, d_inst, d_perm, d_os, d_pos, d_tmp, cfg->n_instances, n, st) != cudaSuccess)
         return ISJL_ERR_CUDA;
@@ -115,6 +117,7 @@ extern "C" isjl_status isjl_sim_run_sweep_noalloc(const isjl_config *cfg, int32_
     std::memset(&a, 0, sizeof(a));
     a.arrival = in->arrival;
     a.o = d_o;
+    a.otrue = d_ot;
     a.perm = d_perm;
     a.osorted = d_os;
     a.posof = d_pos;

@@ -36,7 +36,8 @@ __device__ __forceinline__ T warp_max(T v) {
 // one block per instance
 __global__ void __launch_bounds__(kDeriveThreads)
 derive_kernel(const int32_t *__restrict__ arrival, const int32_t *__restrict__ prompt,
-              const int32_t *__restrict__ output, const int32_t *__restrict__ count, int32_t *__restrict__ o,
+              const int32_t *__restrict__ output, const int32_t *__restrict__ count,
+              const int32_t *__restrict__ slack, int32_t *__restrict__ o, int32_t *__restrict__ otrue,
               InstStats *inst, int32_t n_slots) {
     const int64_t base = (int64_t)blockIdx.x * n_slots;
     int64_t O = 0, Q = 0, sumA = 0;
@@ -45,15 +46,21 @@ derive_kernel(const int32_t *__restrict__ arrival, const int32_t *__restrict__ p
     if (n < 0 || n > n_slots) { invalid = 1; n = 0; }
     for (int i = threadIdx.x; i < n; i += kDeriveThreads) {
         const int32_t a = arrival[base + i], p = prompt[base + i], q = output[base + i];
+        const int32_t e = slack ? slack[base + i] : 0;
         const int64_t oi = (int64_t)p + q;
-        if (a < 0 || p < 0 || q < 0 || (i > 0 && arrival[base + i - 1] > a) || oi > ISJL_MAX_LEN) invalid = 1;
+        const int64_t ui = oi + e;                  // planning length (Robust-ISJL's u_i)
+        if (a < 0 || p < 0 || q < 0 || e < 0 || (i > 0 && arrival[base + i - 1] > a) || ui > ISJL_MAX_LEN)
+            invalid = 1;
         else if (oi < 1) infeasible = 1;
-        const int32_t oc = (oi < 0 || oi > ISJL_MAX_LEN) ? 0 : (int32_t)oi;
-        o[base + i] = oc;
+        const bool ok = oi >= 0 && ui <= ISJL_MAX_LEN && e >= 0;
+        const int32_t oc = ok ? (int32_t)oi : 0;
+        const int32_t uc = ok ? (int32_t)ui : 0;
+        o[base + i] = uc;
+        if (otrue) otrue[base + i] = oc;
         O += oc;
         Q += (int64_t)oc * (oc + 1) / 2;
         sumA += a;
-        maxo = max(maxo, oc);
+        maxo = max(maxo, uc);
         maxA = max(maxA, a);
     }
     O = warp_sum(O); Q = warp_sum(Q); sumA = warp_sum(sumA);
@@ -244,9 +251,10 @@ summarize_kernel(const isjl_record *__restrict__ rec, int64_t n_inst, RunList ru
 }  // namespace
 
 cudaError_t launch_derive(const int32_t *arrival, const int32_t *prompt, const int32_t *output,
-                          const int32_t *count, int32_t *o, InstStats *inst, int64_t n_inst, int32_t n,
-                          cudaStream_t s) {
-    derive_kernel<<<(unsigned)n_inst, kDeriveThreads, 0, s>>>(arrival, prompt, output, count, o, inst, n);
+                          const int32_t *count, const int32_t *slack, int32_t *o, int32_t *otrue,
+                          InstStats *inst, int64_t n_inst, int32_t n, cudaStream_t s) {
+    derive_kernel<<<(unsigned)n_inst, kDeriveThreads, 0, s>>>(arrival, prompt, output, count, slack, o, otrue,
+                                                              inst, n);
     return cudaGetLastError();
 }
 

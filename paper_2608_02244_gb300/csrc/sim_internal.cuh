@@ -17,10 +17,10 @@ constexpr int kRadixThreads = 128;            // threads of the large-n radix so
 
 // Per-instance facts derived once per call (policy independent).
 struct InstStats {
-    int64_t O;        // sum o_i
+    int64_t O;        // sum o_i (true lengths)
     int64_t Q;        // sum o_i (o_i + 1) / 2
     int64_t sumA;     // sum of arrivals
-    int32_t maxo;     // largest o_i
+    int32_t maxo;     // largest planning length u_i (= o_i without slack): KV feasibility
     int32_t maxA;     // largest arrival
     int32_t status;   // ISJL_OK, ISJL_ERR_INVALID_ARG or ISJL_ERR_INFEASIBLE (o_i < 1)
     int32_t n;        // requests of this instance (its first n slots)
@@ -48,7 +48,8 @@ inline int32_t run_beta(int32_t policy, int32_t delta) {
 
 struct SimArgs {
     const int32_t *arrival;    // [N] instance-major
-    const int32_t *o;          // [N] o_i = prompt + output
+    const int32_t *o;          // [N] planning length u_i = prompt + output (+ slack)
+    const int32_t *otrue;      // [N] true length o_i, or null when there is no slack
     const int32_t *perm;       // [N] sorted position -> request index within its instance
     const int32_t *osorted;    // [N] o at each sorted position (non-increasing)
     const int32_t *posof;      // [N] request index -> sorted position
@@ -73,8 +74,8 @@ struct SimArgs {
 
 // host-side launchers (defined in the .cu files)
 cudaError_t launch_derive(const int32_t *arrival, const int32_t *prompt, const int32_t *output,
-                          const int32_t *count, int32_t *o, InstStats *inst, int64_t n_inst, int32_t n,
-                          cudaStream_t s);
+                          const int32_t *count, const int32_t *slack, int32_t *o, int32_t *otrue,
+                          InstStats *inst, int64_t n_inst, int32_t n, cudaStream_t s);
 cudaError_t launch_sort(const int32_t *o, const InstStats *inst, int32_t *perm, int32_t *osorted, int32_t *posof,
                         int32_t *tmp, int64_t n_inst, int32_t n, cudaStream_t s);
 cudaError_t launch_sim(const SimArgs &args, bool epoch, int total_warps, cudaStream_t s);

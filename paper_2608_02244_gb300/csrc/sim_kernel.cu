@@ -51,12 +51,13 @@ struct WarpSmem {
     int32_t *slong;   // [B] long request o_j planned on worker j (1 <= j < n_long)
     int32_t *srem;    // [B] ISJL packing budget left on worker w (Phase ONE only)
     int32_t *spsum;   // [B] ISJL pack sum on worker w (Phase ONE only)
+    int32_t *sres;    // [B] KV reserved by the request running on worker w (its planning length)
     uint32_t *pend0;  // [words0] bit p: sorted position p is pending
     uint32_t *pend1;  // [words1] bit w: pend0[w] != 0
 };
 
 __host__ __device__ inline int smem_words_per_warp(int B, int words0, int words1) {
-    int w = 6 * B + words0 + words1;
+    int w = 7 * B + words0 + words1;
     return (w + 3) & ~3;  // keep every warp's block 16-byte aligned
 }
 
@@ -171,7 +172,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     const int64_t beta = A.runs.beta[run];
     const int64_t kv_cap = A.kv_cap;
     const int32_t *__restrict__ arr = A.arrival + base;
-    const int32_t *__restrict__ oarr = A.o + base;
+    const int32_t *__restrict__ oarr = A.o + base;              // planning lengths (u_i)
+    const int32_t *__restrict__ otru = A.otrue ? A.otrue + base : nullptr;   // true lengths
     const int32_t *__restrict__ perm = A.perm + base;
     const int32_t *__restrict__ osrt = A.osorted + base;
     const int32_t *__restrict__ posof = A.posof + base;
@@ -246,9 +248,10 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         };
         // start request e (length oe) on worker w at step k
         auto start = [&](int e, int oe, int w) {
+            const int oc = otru ? otru[e] : oe;          // it finishes after its true length
             run_cnt++;
-            kv_sum += oe;
-            cmin = min(cmin, k + oe);
+            kv_sum += oe;                                // and reserves its planning length
+            cmin = min(cmin, k + oc);
             peakkv = max(peakkv, kv_sum);
             peakb = max(peakb, run_cnt);
             kv_over = kv_sum > kv_cap;
@@ -257,9 +260,10 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (lane == owner) {
 #pragma unroll
                 for (int r = 0; r < SPL; ++r)
-                    if (r == row) { sa[r] = EPOCH ? k : 0; sc[r] = k + oe; }
+                    if (r == row) { sa[r] = EPOCH ? k : 0; sc[r] = k + oc; }
                 busy |= 1u << row;
-                lane_cmin = min(lane_cmin, k + oe);
+                lane_cmin = min(lane_cmin, k + oc);
+                S.sres[w] = oe;
                 if (EPOCH) { lane_smin = min(lane_smin, k); lane_smax = max(lane_smax, k); }
                 S.sjob[w] = e;
                 if (st_out) st_out[e] = k;
@@ -281,7 +285,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if ((busy >> r & 1u) && sc[r] == c) {
                     fm |= 1u << r;
                     nf++;
-                    of += EPOCH ? sc[r] - sa[r] : sa[r];
+                    of += S.sres[(r << 5) + lane];
                     if (EPOCH) sf += (unsigned)(sa[r] - (c - 65536));
                     if (co_out) co_out[S.sjob[(r << 5) + lane]] = c;
                     sc[r] = INT_MAX;
@@ -716,7 +720,8 @@ sim_kernel(SimArgs A, int64_t n_tasks) {
     S.slong = b + 3 * A.B;
     S.srem = b + 4 * A.B;
     S.spsum = b + 5 * A.B;
-    S.pend0 = reinterpret_cast<uint32_t *>(b + 6 * A.B);
+    S.sres = b + 6 * A.B;
+    S.pend0 = reinterpret_cast<uint32_t *>(b + 7 * A.B);
     S.pend1 = S.pend0 + A.words0;
     const int64_t gwarp = (int64_t)blockIdx.x * kSimWarpsPerBlock + wib;
     for (;;) {

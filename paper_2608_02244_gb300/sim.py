@@ -39,7 +39,7 @@ class isjl_config(ctypes.Structure):
 
 class isjl_instances(ctypes.Structure):
     _fields_ = [("arrival", ctypes.c_void_p), ("prompt", ctypes.c_void_p), ("output", ctypes.c_void_p),
-                ("count", ctypes.c_void_p)]
+                ("count", ctypes.c_void_p), ("slack", ctypes.c_void_p)]
 
 
 class isjl_outputs(ctypes.Structure):
@@ -149,9 +149,10 @@ def _stream_ptr(stream):
     return ctypes.c_void_p(int(stream.cuda_stream))
 
 
-def _instances(arrival, prompt, output, count):
+def _instances(arrival, prompt, output, count, slack=None):
     return isjl_instances(arrival.data_ptr(), prompt.data_ptr(), output.data_ptr(),
-                          count.data_ptr() if count is not None else None)
+                          count.data_ptr() if count is not None else None,
+                          slack.data_ptr() if slack is not None else None)
 
 
 def isjl_sim_run(handle, policy, delta, kv_cap, arrival, prompt, output, records, start=None,
@@ -164,10 +165,10 @@ def isjl_sim_run(handle, policy, delta, kv_cap, arrival, prompt, output, records
 
 
 def isjl_sim_run_sweep(handle, policies, deltas, kv_cap, arrival, prompt, output, records, start=None,
-                       completion=None, stream=None, count=None):
+                       completion=None, stream=None, count=None, slack=None):
     pol = _i32_array([_policy_code(p) for p in policies])
     dl = _i32_array(deltas)
-    ins = _instances(arrival, prompt, output, count)
+    ins = _instances(arrival, prompt, output, count, slack)
     outs = isjl_outputs(records.data_ptr(), start.data_ptr() if start is not None else None,
                         completion.data_ptr() if completion is not None else None)
     return lib().isjl_sim_run_sweep(handle, len(pol), pol, dl, int(kv_cap), ctypes.byref(ins),
@@ -187,7 +188,7 @@ def isjl_sim_run_sweep_host(handle, policies, deltas, kv_cap, h_arrival, h_promp
 
 def isjl_sim_run_sweep_noalloc(n_instances, n_per_instance, B, policies, deltas, kv_cap, arrival, prompt,
                                output, records, start=None, completion=None, c=0.0005, tau=1e-6, p0=0.002,
-                               max_steps=0, flags=FLAG_STEP_KERNEL, stream=None, count=None):
+                               max_steps=0, flags=FLAG_STEP_KERNEL, stream=None, count=None, slack=None):
     """Allocation-free sweep for callers that cannot allocate device memory at the
     point of use (allocator-owned pools, fixed budgets, no-sync sections): the
     library's workspace is a fixed device array shared by all calls, so calls
@@ -197,7 +198,7 @@ def isjl_sim_run_sweep_noalloc(n_instances, n_per_instance, B, policies, deltas,
                       int(max_steps), int(flags))
     pol = _i32_array([_policy_code(p) for p in policies])
     dl = _i32_array(deltas)
-    ins = _instances(arrival, prompt, output, count)
+    ins = _instances(arrival, prompt, output, count, slack)
     outs = isjl_outputs(records.data_ptr(), start.data_ptr() if start is not None else None,
                         completion.data_ptr() if completion is not None else None)
     return lib().isjl_sim_run_sweep_noalloc(ctypes.byref(cfg), len(pol), pol, dl, int(kv_cap), ctypes.byref(ins),
@@ -274,18 +275,18 @@ class Simulator:
         return rec, st, co
 
     def sweep_async(self, arrival, prompt, output, policies, deltas, kv_cap, per_request=False, stream=None,
-                    counts=None):
+                    counts=None, slack=None):
         """Launch a sweep on device-resident int32 tensors; returns output tensors."""
         rec, st, co = self.buffers(len(policies), per_request)
         if per_request:
             st.fill_(-1)
             co.fill_(-1)
         _check(isjl_sim_run_sweep(self.handle, policies, deltas, kv_cap, arrival, prompt, output, rec, st, co,
-                                  stream, counts), "isjl_sim_run_sweep")
+                                  stream, counts, slack), "isjl_sim_run_sweep")
         return rec, st, co
 
     def sweep(self, arrival, prompt, output, policies, deltas, kv_cap, per_request=False, stream=None,
-              counts=None):
+              counts=None, slack=None):
         """Run a sweep and return numpy results: records (n_runs, n_inst), start and
         completion (n_runs, n_inst, n) or None, per-run summaries, device status."""
         torch = self.torch
@@ -296,7 +297,8 @@ class Simulator:
 
         a, p, o = dev(arrival), dev(prompt), dev(output)
         cnt = dev(counts) if counts is not None else None
-        rec, st, co = self.sweep_async(a, p, o, policies, deltas, kv_cap, per_request, stream, cnt)
+        sl = dev(slack) if slack is not None else None
+        rec, st, co = self.sweep_async(a, p, o, policies, deltas, kv_cap, per_request, stream, cnt, sl)
         status, summ = isjl_sim_metrics(self.handle)
         R = len(policies)
         out = {

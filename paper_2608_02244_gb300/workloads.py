@@ -44,6 +44,7 @@ class Workload:
     policies: tuple = ("fcfs", "ljf", "isjl")
     online: bool = False
     ragged: bool = False  # instances use a variable number of their slots (see counts)
+    robust: bool = False  # comes with an upper-bound slack array (length predictions u = o + slack)
     note: str = ""
     c: float = 0.0005   # fixed cost per service step (Section 5 experiment)
     tau: float = 1e-6   # cost per unit of max-driven footprint
@@ -77,6 +78,14 @@ WORKLOADS = {
     6: Workload(6, "profit-experiment", 10_000, 400, 6000, B=(50,), kv_caps=(KV_INF,),
                 deltas=(50, 100, 150, 250, 300, 400, 500), ragged=True,
                 note="400 offered, o ~ U{1..1000}, bucketed acceptance; accepted requests at t=0"),
+    # Section 3.3 (prediction intervals): the instances of workloads 2 and 3 with an upper-bound
+    # slack e_i = u_i - o_i drawn per request
+    7: Workload(7, "tiny-robust", 4096, 6, 7000, B=(2, 3), kv_caps=(16, KV_INF),
+                deltas=(0, 1, 2, 4, DELTA_INF), policies=("isjl",), robust=True,
+                note="n=6 at t=0; prompt U[1,4]; output U[1,8]; slack U{0..3}"),
+    8: Workload(8, "online-robust", 10_000, 1_000, 8000, B=(256,), kv_caps=(200_000,),
+                deltas=(16, 64, 256, 1024, DELTA_INF), online=True, robust=True,
+                note="workload 3's distributions; slack = rint(output * U[0, 0.5])"),
 }
 
 
@@ -137,13 +146,25 @@ def _draw_chunk(wl: Workload, chunk: int, rows: int, replica: int = 0):
         for r in range(rows):                       # accepted requests first, in offer order
             acc = offered[r][keep[r]]
             output[r, :acc.size] = acc
-        return arrival, prompt, output, count
+        return arrival, prompt, output, count, None
+    elif wl.wid == 7:
+        arrival = np.zeros(shape, np.int32)
+        prompt = rng.integers(1, 5, size=shape, dtype=np.int32)
+        output = rng.integers(1, 9, size=shape, dtype=np.int32)
+        slack = rng.integers(0, 4, size=shape, dtype=np.int32)
+        return arrival, prompt, output, None, slack
+    elif wl.wid == 8:
+        arrival = _poisson_arrivals(rng, shape, 2.0)
+        prompt = _lognormal_int(rng, shape, 512, 1.0, 16, 4096)
+        output = _lognormal_int(rng, shape, 256, 1.2, 1, 2048)
+        slack = np.rint(output * rng.uniform(0.0, 0.5, size=shape)).astype(np.int32)
+        return arrival, prompt, output, None, slack
     else:  # pragma: no cover
         raise ValueError(f"unknown workload {wl.wid}")
-    return arrival, prompt, output, None
+    return arrival, prompt, output, None, None
 
 
-def generate(wid: int, instances=None, replica: int = 0, with_counts: bool = False):
+def generate(wid: int, instances=None, replica: int = 0, with_counts: bool = False, with_slack: bool = False):
     """Return (arrival, prompt, output), each int32 of shape (len(instances), n).
 
     ``instances`` is None (all instances), an int m (the first m) or an
@@ -151,7 +172,9 @@ def generate(wid: int, instances=None, replica: int = 0, with_counts: bool = Fal
     requested.  ``replica`` r > 0 draws an independent set of the same shape
     (seed sequence [seed, chunk, r]); multi-GPU runs give rank r replica r.
     ``with_counts`` appends the per-instance request counts (all n except for
-    ragged workloads, whose instance i uses its first counts[i] slots).
+    ragged workloads, whose instance i uses its first counts[i] slots);
+    ``with_slack`` then appends the upper-bound slack array (zeros unless the
+    workload is robust).
     """
     wl = WORKLOADS[wid]
     if instances is None:
@@ -166,6 +189,7 @@ def generate(wid: int, instances=None, replica: int = 0, with_counts: bool = Fal
     n = wl.n_per_instance
     out = [np.empty((ids.size, n), np.int32) for _ in range(3)]
     cnt = np.empty(ids.size, np.int32)
+    slk = np.zeros((ids.size, n), np.int32)
     chunks = ids // per
     for c in np.unique(chunks):
         sel = np.nonzero(chunks == c)[0]
@@ -176,9 +200,14 @@ def generate(wid: int, instances=None, replica: int = 0, with_counts: bool = Fal
         for k in range(3):
             out[k][sel] = arrs[k][ids[sel] % per]
         cnt[sel] = arrs[3][ids[sel] % per] if arrs[3] is not None else n
+        if arrs[4] is not None:
+            slk[sel] = arrs[4][ids[sel] % per]
+    res = tuple(out)
     if with_counts:
-        return tuple(out) + (cnt,)
-    return tuple(out)
+        res = res + (cnt,)
+    if with_slack:
+        res = res + (slk,)
+    return res
 
 
 def custom(arrival, prompt, output):

@@ -44,7 +44,8 @@ EXAMPLES = parse_examples(os.path.join(GOLDEN, "worked_examples.txt"))
 @pytest.mark.parametrize("ex", EXAMPLES, ids=[e["name"] for e in EXAMPLES])
 def test_hand_derived_schedules(oracle_mod, ex):
     z = np.zeros_like(ex["o"])
-    rec, st, co = oracle_mod.run(ex["policy"], ex["B"], ex["delta"], ex["kv"], ex["arrival"], z, ex["o"])
+    rec, st, co = oracle_mod.run(ex["policy"], ex["B"], ex["delta"], ex["kv"], ex["arrival"], z, ex["o"],
+                                 slack=ex.get("slack"))
     assert rec["status"] == 0
     np.testing.assert_array_equal(st, ex["start"])
     np.testing.assert_array_equal(co, ex["completion"])

@@ -40,18 +40,18 @@ def assert_records_equal(g, r, ctx=""):
 
 
 def run_both(S, O, a, p, o, B, policies, deltas, kv, epoch, per_request=True, max_steps=0, check=True,
-             counts=None):
+             counts=None, slack=None):
     n_inst, n = a.shape
     sm = S.Simulator(n_inst, n, B, max_steps=max_steps, epoch=epoch)
     try:
-        res = sm.sweep(a, p, o, policies, deltas, kv, per_request=per_request, counts=counts)
+        res = sm.sweep(a, p, o, policies, deltas, kv, per_request=per_request, counts=counts, slack=slack)
     finally:
         sm.close()
     assert res["launches"] == 4
     if check:
         for i, (pol, d) in enumerate(zip(policies, deltas)):
             rec, st, co = O.run(pol, B, d, kv, a, p, o, max_steps=max_steps, per_request=per_request,
-                                counts=counts)
+                                counts=counts, slack=slack)
             assert_records_equal(res["records"][i], rec, f"{pol} d={d} epoch={epoch}")
             if per_request:
                 np.testing.assert_array_equal(res["start"][i], st, err_msg=f"start {pol} {d}")
@@ -186,6 +186,27 @@ def test_profit_experiment_workload_ragged(S, O, epoch):
 
 
 @pytest.mark.parametrize("epoch", EPOCHS)
+@pytest.mark.parametrize("B", [2, 3])
+def test_tiny_robust_workload(S, O, epoch, B):
+    """Robust-ISJL: plans with u = o + slack, serves o (Section 3.3)."""
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o, e = W.generate(7, with_slack=True)
+    pols = ["isjl"] * 5 + ["fcfs", "ljf", "sjf", "isjl_beta"]
+    ds = [0, 1, 2, 4, INF, 0, 0, 0, 2]
+    for kv in (16, INF):
+        run_both(S, O, a, p, o, B, pols, ds, kv, epoch, slack=e)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_online_robust_workload_subset(S, O, epoch):
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o, e = W.generate(8, 12, with_slack=True)
+    pols = ["fcfs", "ljf", "isjl", "isjl", "isjl", "sjf", "isjl_beta"]
+    ds = [0, 0, 16, 256, INF, 0, 256]
+    run_both(S, O, a, p, o, 256, pols, ds, 200_000, epoch, slack=e)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
 def test_ragged_counts_edges(S, O, epoch):
     """Empty instances, full instances, and an out-of-range count (INVALID_ARG)."""
     rng = np.random.default_rng(9)
@@ -196,6 +217,9 @@ def test_ragged_counts_edges(S, O, epoch):
     cnt = np.array([0, n, 1, 33, 0, 64], np.int32)
     run_both(S, O, a, p, o, 8, ["fcfs", "ljf", "isjl", "isjl", "sjf", "isjl_beta"], [0, 0, 4, INF, 0, 4], 200, epoch,
              counts=cnt)
+    e = rng.integers(0, 15, (6, n)).astype(np.int32)        # with predictions as well
+    run_both(S, O, a, p, o, 8, ["fcfs", "ljf", "isjl", "isjl", "sjf", "isjl_beta"], [0, 0, 4, INF, 0, 4], 300, epoch,
+             counts=cnt, slack=e)
     bad = cnt.copy()
     bad[2] = n + 1
     res = run_both(S, O, a, p, o, 8, ["isjl"], [4], 200, epoch, counts=bad, check=False)
