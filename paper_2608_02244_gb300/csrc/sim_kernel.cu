@@ -278,19 +278,24 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         // requests completing at step c leave their workers
         auto retire = [&](int32_t c) {
             uint32_t fm = 0u;
-            int nf = 0, of = 0;
             unsigned sf = 0u;   // sum of (start - (c - 65536)) over finishing requests (epoch kernel)
 #pragma unroll
             for (int r = 0; r < SPL; ++r) {
-                if ((busy >> r & 1u) && sc[r] == c) {
-                    fm |= 1u << r;
-                    nf++;
-                    of += S.sres[(r << 5) + lane];
+                const bool f = sc[r] == c;                   // idle slots hold INT_MAX
+                fm |= (uint32_t)f << r;
+                if (f) {
                     if (EPOCH) sf += (unsigned)(sa[r] - (c - 65536));
-                    if (co_out) co_out[S.sjob[(r << 5) + lane]] = c;
                     sc[r] = INT_MAX;
-                    if (!EPOCH) sa[r] = kIdle + c - 1;   // sentinel of the step just served
+                    if (!EPOCH) sa[r] = kIdle + c - 1;       // sentinel of the step just served
                 }
+            }
+            // per finishing request (usually one per warp): outputs and its KV release
+            int nf = 0, of = 0;
+            for (uint32_t m = fm; m; m &= m - 1u) {
+                const int w = ((__ffs(m) - 1) << 5) + lane;
+                nf++;
+                of += S.sres[w];
+                if (co_out) co_out[S.sjob[w]] = c;
             }
             busy &= ~fm;
             if (fm) recompute_lane();
