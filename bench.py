@@ -9,8 +9,10 @@ clipped [16, 4096]; output lognormal(ln 256, 1.2) clipped [1, 2048]), KV cap
 delta in {16, 64, 256, 1024, inf} (7 runs per instance), per-request start and
 completion steps written out.  A batch-step is a simulated step whose batch
 is nonempty; value = sum over (instance, run) of T_busy per second.
+--workload picks another workload's run grid (GRIDS below) for the same
+measurement; the default line is the online delta-sweep.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--kernel step|epoch]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--kernel step|epoch] [--workload 3|4|5|6|8]
   python bench.py --impl reference ...     (the CPU oracle on host cores)
 
 Multi-GPU (torchrun): rank r simulates its own replica of the workload
@@ -38,10 +40,17 @@ from paper_2608_02244_gb300 import workloads as W  # noqa: E402
 
 METRIC = "simulated batch-steps/sec on 1 GB300 (ISJL Δ-sweep); % of HBM/int roofline"
 UNIT = "batch-steps/s"
-WID = 3
 INF = W.DELTA_INF
-POLICIES = ["fcfs", "ljf", "isjl", "isjl", "isjl", "isjl", "isjl"]
-DELTAS = [0, 0, 16, 64, 256, 1024, INF]
+DEFAULT_WID = 3
+# per workload: (policies, fairness budgets, oracle instances per host core for
+# the CPU baseline sample: one to two seconds of oracle work per core)
+GRIDS = {
+    3: (["fcfs", "ljf", "isjl", "isjl", "isjl", "isjl", "isjl"], [0, 0, 16, 64, 256, 1024, INF], 40),
+    4: (["fcfs", "ljf", "isjl", "isjl", "isjl"], [0, 0, 32, 128, 512], 400),
+    5: (["fcfs", "ljf", "isjl"], [0, 0, 256], 1),
+    6: (["fcfs", "ljf"] + ["isjl"] * 7, [0, 0, 50, 100, 150, 250, 300, 400, 500], 400),
+    8: (["fcfs", "ljf", "isjl", "isjl", "isjl", "isjl", "isjl"], [0, 0, 16, 64, 256, 1024, INF], 40),
+}
 # int32 ALU lanes per SM on GB300 (4 SM sub-partitions x 32 lanes) and SM count
 ALU_LANES_PER_SM = 128
 # algorithmic integer work of the per-step kernel: per token-advance
@@ -55,13 +64,13 @@ OPS_PER_BATCH_STEP = 6
 SIM_DRAM_BYTES_PER_LAUNCH = 576.7e6 * 10_000 / 4_096
 
 
-def workload_config(kernel, wl, flush):
+def workload_config(kernel, wl, n_inst, policies, deltas, flush):
+    kv = "none" if wl.kv_caps[0] == W.KV_INF else wl.kv_caps[0]
     return {
-        "workload": f"online-delta-sweep: {wl.n_instances} instances x {wl.n_per_instance} requests, "
-                    "Poisson arrivals mean gap 2; prompt LN(ln512,1) [16,4096]; output LN(ln256,1.2) [1,2048]",
-        "B": wl.B[0], "kv_cap": wl.kv_caps[0], "policies": POLICIES,
-        "deltas": ["inf" if d == INF else d for d in DELTAS],
-        "runs_per_instance": len(POLICIES), "per_request_outputs": True,
+        "workload": f"{wl.name}: {n_inst} instances x {wl.n_per_instance} requests, {wl.note}",
+        "B": wl.B[0], "kv_cap": kv, "policies": policies,
+        "deltas": ["inf" if d == INF else d for d in deltas],
+        "runs_per_instance": len(policies), "per_request_outputs": True,
         "kernel": kernel, "l2": flush,
     }
 
@@ -113,24 +122,36 @@ class ClockSampler:
 # ------------------------------------------------------------ CPU oracle ----
 def _oracle_chunk(args):
     """Worker: run the oracle on a block of instances; returns (sum T_busy, sum token_adv)."""
-    a, p, o, B, kv = args
+    a, p, o, cnt, slack, B, kv, policies, deltas = args
     sys.path.insert(0, ROOT)
     from oracle import oracle as O
     tb = tok = 0
-    for pol, d in zip(POLICIES, DELTAS):
-        rec, _, _ = O.run(pol, B, d, kv, a, p, o, per_request=False)
+    for pol, d in zip(policies, deltas):
+        rec, _, _ = O.run(pol, B, d, kv, a, p, o, per_request=False, counts=cnt, slack=slack)
         tb += int(rec["T_busy"].sum())
         tok += int(rec["token_adv"].sum())
     return tb, tok
 
 
-def oracle_timed(a, p, o, B, kv, cores, pool):
+def oracle_timed(inputs, B, kv, policies, deltas, cores, pool):
+    """Oracle over `inputs` split into one block per core; (sum T_busy, sum
+    token advances, wall seconds, blocks)."""
+    a, p, o, cnt, slack = inputs
     chunks = [x for x in np.array_split(np.arange(len(a)), cores) if len(x)]
-    jobs = [(a[c], p[c], o[c], B, kv) for c in chunks]
+    jobs = [(a[c], p[c], o[c], None if cnt is None else cnt[c], None if slack is None else slack[c],
+             B, kv, policies, deltas) for c in chunks]
     t = time.perf_counter()
     res = pool.map(_oracle_chunk, jobs)
     dt = time.perf_counter() - t
-    return sum(r[0] for r in res), sum(r[1] for r in res), dt
+    return sum(r[0] for r in res), sum(r[1] for r in res), dt, len(jobs)
+
+
+def host_inputs(wid, count, replica=0):
+    """(arrival, prompt, output, counts or None, slack or None) of the first
+    `count` instances; counts only for ragged workloads, slack only for robust."""
+    wl = W.WORKLOADS[wid]
+    a, p, o, cnt, slack = W.generate(wid, count, replica=replica, with_counts=True, with_slack=True)
+    return a, p, o, (cnt if wl.ragged else None), (slack if wl.robust else None)
 
 
 def cpu_model():
@@ -168,18 +189,19 @@ def reference_arm(args):
     world, rank, _ = dist_env()
     if rank != 0:
         return 0
-    wl = W.WORKLOADS[WID]
+    wl = W.WORKLOADS[args.workload]
+    policies, deltas, per_core = GRIDS[args.workload]
+    per_core = max(1, per_core * 3 // 10)
     cores = os.cpu_count() or 1
-    per_core = 12
-    a, p, o = W.generate(WID, cores * per_core)
+    inputs = host_inputs(args.workload, cores * per_core)
     ctx = mp.get_context("spawn")
     with ctx.Pool(cores) as pool:
         for _ in range(args.warmup):
-            oracle_timed(a, p, o, wl.B[0], wl.kv_caps[0], cores, pool)
+            oracle_timed(inputs, wl.B[0], wl.kv_caps[0], policies, deltas, cores, pool)
         tb_tot = tok_tot = 0
         t_tot = 0.0
         for _ in range(args.steps):
-            tb, tok, dt = oracle_timed(a, p, o, wl.B[0], wl.kv_caps[0], cores, pool)
+            tb, tok, dt, _ = oracle_timed(inputs, wl.B[0], wl.kv_caps[0], policies, deltas, cores, pool)
             tb_tot += tb
             tok_tot += tok
             t_tot += dt
@@ -188,9 +210,11 @@ def reference_arm(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t_tot / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
-        "data": "synthetic", "config": workload_config("cpu-oracle", wl, "n/a (CPU)"),
+        "data": "synthetic",
+        "config": workload_config("cpu-oracle", wl, wl.n_instances, policies, deltas, "n/a (CPU)"),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                         "sample": f"first {cores * per_core} of {wl.n_instances} instances x 7 runs per step",
+                         "sample": f"first {cores * per_core} of {wl.n_instances} instances x "
+                                   f"{len(policies)} runs per step",
                          "cpu": cpu_model()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "token_advances_per_s": tok_tot / t_tot,
@@ -206,6 +230,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--kernel", choices=["step", "epoch"], default="step")
+    ap.add_argument("--workload", type=int, choices=sorted(GRIDS), default=DEFAULT_WID)
     ap.add_argument("--instances", type=int, default=0, help="use only the first N instances (profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -215,14 +240,16 @@ def main():
         return reference_arm(args)
 
     world, rank, local = dist_env()
-    wl = W.WORKLOADS[WID]
-    n_inst = args.instances or wl.n_instances
+    wid = args.workload
+    wl = W.WORKLOADS[wid]
+    policies, deltas, per_core = GRIDS[wid]
+    n_inst = min(args.instances or wl.n_instances, wl.n_instances)
     B, kv = wl.B[0], wl.kv_caps[0]
 
     # the oracle pool starts before the first CUDA call (spawned workers)
     pool = None
     cores = os.cpu_count() or 1
-    if rank == 0 and world >= 1 and not args.no_cpu_baseline:
+    if rank == 0 and not args.no_cpu_baseline:
         pool = mp.get_context("spawn").Pool(cores)
 
     import torch
@@ -233,22 +260,25 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     from paper_2608_02244_gb300 import sim
 
-    a_h, p_h, o_h = W.generate(WID, n_inst, replica=rank)
-    a = torch.from_numpy(a_h).cuda()
-    p = torch.from_numpy(p_h).cuda()
-    o = torch.from_numpy(o_h).cuda()
+    a_h, p_h, o_h, c_h, e_h = host_inputs(wid, n_inst, replica=rank)
+    a, p, o = (torch.from_numpy(x).cuda() for x in (a_h, p_h, o_h))
+    cnt = torch.from_numpy(c_h).cuda() if c_h is not None else None
+    slk = torch.from_numpy(e_h).cuda() if e_h is not None else None
     epoch = args.kernel == "epoch"
     S = sim.Simulator(n_inst, wl.n_per_instance, B, wl.c, wl.tau, wl.p0, epoch=epoch, timing=True)
     flush = torch.empty(64 * 2**20, dtype=torch.int32, device="cuda")   # 256 MiB > 129 MB L2
     stream = torch.cuda.current_stream()
 
+    def sweep(simr):
+        return simr.sweep_async(a, p, o, policies, deltas, kv, per_request=True, counts=cnt, slack=slk)
+
     # warm-up (also yields the deterministic per-step unit counts)
     for _ in range(max(args.warmup, 1)):
-        S.sweep_async(a, p, o, POLICIES, DELTAS, kv, per_request=True)
+        sweep(S)
     st, summ = sim.isjl_sim_metrics(S.handle)
     if st != 0:
         raise RuntimeError(f"device status {st}: {sim.isjl_status_string(st)}")
-    runs = [sim.summary_to_dict(summ[i]) for i in range(len(POLICIES))]
+    runs = [sim.summary_to_dict(summ[i]) for i in range(len(policies))]
     busy_per_step = sum(r["T_busy"] for r in runs)
     tok_per_step = sum(r["token_adv"] for r in runs)
     launches_per_step = sim.isjl_sim_last_launches(S.handle)
@@ -274,7 +304,7 @@ def main():
         for k in range(args.steps):
             flush.zero_()
             ev0[k].record(stream)
-            simr.sweep_async(a, p, o, POLICIES, DELTAS, kv, per_request=True)
+            sweep(simr)
             ev1[k].record(stream)
             sim_ms.append(sim.isjl_sim_kernel_times(simr.handle)[2])   # waits for this step's events
         torch.cuda.synchronize()
@@ -294,9 +324,9 @@ def main():
     if not args.no_epoch:
         S2 = sim.Simulator(n_inst, wl.n_per_instance, B, wl.c, wl.tau, wl.p0, epoch=not epoch, timing=True)
         for _ in range(max(args.warmup, 1)):
-            S2.sweep_async(a, p, o, POLICIES, DELTAS, kv, per_request=True)
+            sweep(S2)
         st2, summ2 = sim.isjl_sim_metrics(S2.handle)
-        busy2 = sum(summ2[i].T_busy for i in range(len(POLICIES)))
+        busy2 = sum(summ2[i].T_busy for i in range(len(policies)))
         if st2 != 0 or busy2 != busy_per_step:
             raise RuntimeError("kernel variants disagree")
         step2, sim2, _ = timed_steps(S2)
@@ -305,17 +335,18 @@ def main():
                  "ms_per_step": sum(step2) / args.steps, "sim_ms_per_launch": sum(sim2) / len(sim2)}
         S2.close()
 
-    # e2e through the host-memory entry point: H2D of the inputs, sweep, D2H of the records
+    # e2e through the host-memory entry point: H2D of the inputs, sweep, D2H of
+    # the records (that entry point takes no counts or slack arrays)
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and c_h is None and e_h is None:
         pa, pp, po = (torch.from_numpy(x).pin_memory() for x in (a_h, p_h, o_h))
-        hrec = torch.empty(len(POLICIES) * n_inst * sim.RECORD_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
-        sim.isjl_sim_run_sweep_host(S.handle, POLICIES, DELTAS, kv, pa, pp, po, hrec)   # warm
+        hrec = torch.empty(len(policies) * n_inst * sim.RECORD_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
+        sim.isjl_sim_run_sweep_host(S.handle, policies, deltas, kv, pa, pp, po, hrec)   # warm
         torch.cuda.synchronize()
         e2e_ms = []
         for _ in range(args.steps):
             t0 = time.perf_counter()
-            rc = sim.isjl_sim_run_sweep_host(S.handle, POLICIES, DELTAS, kv, pa, pp, po, hrec)
+            rc = sim.isjl_sim_run_sweep_host(S.handle, policies, deltas, kv, pa, pp, po, hrec)
             e2e_ms.append(1e3 * (time.perf_counter() - t0))
             if rc != 0:
                 raise RuntimeError(f"host sweep status {rc}")
@@ -345,9 +376,10 @@ def main():
     else:
         ops = OPS_PER_TOKEN_ADVANCE * tok_per_step + OPS_PER_BATCH_STEP * busy_per_step
         achieved = ops / (sim_avg_ms / 1e3) / 1e12
+        full = wid == DEFAULT_WID and n_inst == wl.n_instances
         roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s",
                     "frac": achieved / peak_tops,
-                    "traffic": SIM_DRAM_BYTES_PER_LAUNCH if n_inst == wl.n_instances else None,
+                    "traffic": SIM_DRAM_BYTES_PER_LAUNCH if full else None,
                     "kernel": "sim_kernel (step)", "ops_per_launch": ops,
                     "peak_basis": f"{sms} SMs x {ALU_LANES_PER_SM} int32 lanes x {sm_mhz:.0f} MHz (median SM clock "
                                   "sampled during the timed steps)",
@@ -355,21 +387,20 @@ def main():
 
     cpu = None
     if pool is not None:
-        per_core = 40          # about 20 s of single-core oracle work in total
         sample_n = min(n_inst, cores * per_core)
-        tb, tok, dt = oracle_timed(a_h[:sample_n], p_h[:sample_n], o_h[:sample_n], B, kv, cores, pool)
+        tb, tok, dt, used = oracle_timed(host_inputs(wid, sample_n, replica=rank), B, kv, policies, deltas,
+                                         cores, pool)
         pool.close()
-        cpu = {"value": tb / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"first {sample_n} of {n_inst} instances x {len(POLICIES)} runs ({dt:.1f} s wall)",
+        cpu = {"value": tb / dt, "unit": UNIT, "cores": used, "kind": "oracle",
+               "sample": f"first {sample_n} of {n_inst} instances x {len(policies)} runs ({dt:.1f} s wall)",
                "cpu": cpu_model()}
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": t_ms_all / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
-        "config": workload_config(args.kernel, W.WORKLOADS[WID] if n_inst == wl.n_instances else
-                                  W.Workload(3, "subset", n_inst, wl.n_per_instance, wl.seed, wl.B, wl.kv_caps,
-                                             wl.deltas), "flushed between steps (256 MiB write, outside the events)"),
+        "config": workload_config(args.kernel, wl, n_inst, policies, deltas,
+                                  "flushed between steps (256 MiB write, outside the events)"),
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": ({"value": units_all / (e2e_ms_all / 1e3) / args.steps, "unit": UNIT,
@@ -377,7 +408,7 @@ def main():
         "gpu_launches": launches_per_step * args.steps,
         "clocks": {"sm_mhz": clocks.get("sm_mhz"), "sm_max_mhz": clocks.get("sm_max_mhz"),
                    "reasons": clocks.get("reasons")},
-        "instances_per_s": world * n_inst * len(POLICIES) * args.steps / (t_ms_all / 1e3),
+        "instances_per_s": world * n_inst * len(policies) * args.steps / (t_ms_all / 1e3),
         "token_advances_per_s": tok_per_step * world * args.steps / (t_ms_all / 1e3),
         "kernel_ms": {"sim": sim_avg_ms},
         "other_kernel": other,

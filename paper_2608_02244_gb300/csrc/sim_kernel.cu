@@ -11,14 +11,16 @@
 //             (Section 5, Eq. batch-cost-progress and the decomposition)
 //
 // Layout.  Worker (batch slot) w lives in lane w % 32, register row w / 32,
-// so a warp holds B <= 32 * SPL workers.  The step kernel advances every
-// slot each step, straight-line: an idle slot carries the sentinel progress
-// IDLE + k, which is below every real progress as a signed value, above it as
-// an unsigned value, and known, so the step's max (signed), min (unsigned) and
-// sum (corrected by the idle count) need no per-slot predicate.  Values that
-// change only at events (next arrival, earliest completion, start range, KV
-// reservation) are kept as warp-uniform scalars, so a step without an event
-// runs no warp reduction beyond the three of the step cost.  The pending
+// so a warp holds B <= 32 * SPL workers.  The step kernel advances, each
+// step, every slot of the rows that hold a running worker (a per-row-count
+// instantiation of the step loop), straight-line: an idle slot carries a
+// progress below 0 as a signed value and at least 2^31 as an unsigned one, so
+// the step's max (signed) and min (unsigned) need no per-slot predicate.  The
+// sum of progress over all steps is added per request when it leaves
+// (a (a + 1) / 2 for progress a).  Values that change only at events (next
+// arrival, earliest completion, start range, KV reservation) are kept as
+// warp-uniform scalars, so the steps between two events run no branch and
+// no warp reduction beyond the two of the step cost.  The pending
 // queue is a bitset over the instance's request positions sorted by
 // (o desc, index asc) -- the longest pending request is the lowest set bit --
 // with a summary word per 32 words, in shared memory.  ISJL plans are
@@ -70,6 +72,58 @@ __device__ __forceinline__ int lowest_worker(uint32_t m, int lane) {
 __device__ __forceinline__ int highest_worker(uint32_t m, int lane) {
     const int v = m ? ((31 - __clz(m)) << 5) + lane : -1;
     return __reduce_max_sync(kFull, v);
+}
+
+// a row count as a type, for the step loop's per-row-count instantiations
+template <int N> struct RowCount { static constexpr int value = N; };
+
+// Row counts the step loop is instantiated for, per SPL (ascending).  The
+// loop advances the smallest of them covering every running worker; a few
+// classes keep the kernel small (measured: powers of two for SPL = 8, even
+// counts for SPL = 16), and its steps are unrolled by two.
+template <int SPL> struct RowClasses;
+template <> struct RowClasses<1> {
+    static constexpr int n = 1;
+    __host__ __device__ static constexpr int at(int i) { constexpr int v[1] = {1}; return v[i]; }
+};
+template <> struct RowClasses<2> {
+    static constexpr int n = 2;
+    __host__ __device__ static constexpr int at(int i) { constexpr int v[2] = {1, 2}; return v[i]; }
+};
+template <> struct RowClasses<4> {
+    static constexpr int n = 4;
+    __host__ __device__ static constexpr int at(int i) { constexpr int v[4] = {1, 2, 3, 4}; return v[i]; }
+};
+template <> struct RowClasses<8> {
+    static constexpr int n = 4;
+    __host__ __device__ static constexpr int at(int i) { constexpr int v[4] = {1, 2, 4, 8}; return v[i]; }
+};
+template <> struct RowClasses<16> {
+    static constexpr int n = 8;
+    __host__ __device__ static constexpr int at(int i) { constexpr int v[8] = {2, 4, 6, 8, 10, 12, 14, 16}; return v[i]; }
+};
+
+// rows advanced when the highest row holding a running worker is t - 1 (t = 0: none)
+template <int SPL>
+__device__ __forceinline__ int row_class(int t) {
+    using C = RowClasses<SPL>;
+    if (t <= 0) return 0;
+    int r = SPL;
+#pragma unroll
+    for (int i = C::n - 1; i >= 0; --i) if (C::at(i) >= t) r = C::at(i);
+    return r;
+}
+// call f(RowCount<rows>{}) for rows one of RowClasses<SPL> (indices LO..HI), by a tree of uniform branches
+template <int SPL, int LO, int HI, class F>
+__device__ __forceinline__ void dispatch_rows(int rows, F &f) {
+    using C = RowClasses<SPL>;
+    if constexpr (LO == HI) {
+        f(RowCount<C::at(LO)>{});
+    } else {
+        constexpr int MID = (LO + HI) / 2;
+        if (rows <= C::at(MID)) dispatch_rows<SPL, LO, MID>(rows, f);
+        else dispatch_rows<SPL, MID + 1, HI>(rows, f);
+    }
 }
 
 // acc += a * b into a 64-bit accumulator with one wide multiply-add
@@ -188,8 +242,11 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     // every schedule ends by sum o + max arrival; the idle sentinel needs steps < 2^30
     if (status == ISJL_OK && is.O + (int64_t)is.maxA + 1 >= (int64_t)(1 << 30)) status = ISJL_ERR_INVALID_ARG;
 
-    // W = sum |S| max r; R = sum over steps of sum r (E = W - R at the end)
-    int64_t W = 0, R = 0, E = 0, sumc = 0, sumext = 0, peakkv = 0;
+    // W = sum over steps of |S| max r; E = W - R, where R = sum over steps of
+    // sum r equals the sum over served requests of a (a + 1) / 2 for their
+    // progress a (one token per step from 1), so the step kernel adds it per
+    // request in lane_R (the decomposition W = Q + E of Section 5)
+    int64_t W = 0, lane_R = 0, E = 0, sumc = 0, sumext = 0, peakkv = 0;
     int32_t Tb = 0, tok = 0, maxext = 0, viol = 0, peakb = 0, Tmake = 0, kvviol = 0;
 
     if (status == ISJL_OK && n > 0) {
@@ -212,6 +269,9 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         const int32_t alpha32 = (int32_t)min(alpha, (int64_t)INT_MAX);
 
         int32_t k = 0, rel = 0, fcfs = 0, done = 0, run_cnt = 0, pend = 0;
+        // step kernel: register rows [0, adv_rows) are advanced each step; every
+        // running worker lies in them, and their idle slots hold the sentinel
+        int adv_rows = 0;
         int64_t kv_sum = 0, sum_st = 0;
         // the next 32 unreleased requests (from win_base): arrival and sorted position, per lane
         int32_t win_base = 0, win_a = INT_MAX, win_p = 0;
@@ -257,6 +317,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             kv_over = kv_sum > kv_cap;
             if (EPOCH) { sum_st += k; smin = min(smin, k); smax = k; }
             const int owner = w & 31, row = w >> 5;
+            if (!EPOCH && row >= adv_rows) adv_rows = row_class<SPL>(row + 1);
             if (lane == owner) {
 #pragma unroll
                 for (int r = 0; r < SPL; ++r)
@@ -267,12 +328,6 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (EPOCH) { lane_smin = min(lane_smin, k); lane_smax = max(lane_smax, k); }
                 S.sjob[w] = e;
                 if (st_out) st_out[e] = k;
-            }
-            if (!EPOCH && run_cnt == 1) {
-                // first start after an empty batch: idle slots take the current sentinel
-#pragma unroll
-                for (int r = 0; r < SPL; ++r)
-                    if (!(busy >> r & 1u)) sa[r] = kIdle + k - 1;
             }
         };
         // requests completing at step c leave their workers
@@ -286,7 +341,11 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (f) {
                     if (EPOCH) sf += (unsigned)(sa[r] - (c - 65536));
                     sc[r] = INT_MAX;
-                    if (!EPOCH) sa[r] = kIdle + c - 1;       // sentinel of the step just served
+                    if (!EPOCH) {
+                        const uint32_t a = (uint32_t)sa[r];   // its length; a (a + 1) < 2^32
+                        mad_wide(lane_R, (a * (a + 1u)) >> 1, 1u);
+                        sa[r] = kIdle;
+                    }
                 }
             }
             // per finishing request (usually one per warp): outputs and its KV release
@@ -299,6 +358,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             }
             busy &= ~fm;
             if (fm) recompute_lane();
+            if (!EPOCH) adv_rows = row_class<SPL>((int)__reduce_max_sync(kFull, 32u - (unsigned)__clz((int)busy)));
             nf = (int)__reduce_add_sync(kFull, (unsigned)nf);
             of = (int)__reduce_add_sync(kFull, (unsigned)of);
             if (EPOCH)   // starts are within 65535 steps of c, so the offsets fit 32 bits
@@ -580,11 +640,38 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             }
         };
 
+        // steps k .. k + L - 1 with no event: advance rows [0, NR), which hold
+        // every running worker, and add each step's cost (max r and min r by
+        // warp reductions; idle slots hold a value below 0 as a signed number
+        // and at least 2^31 as an unsigned one, so they lose both)
+        auto plain_steps = [&](auto nr_tag, int L) {
+            constexpr int NR = decltype(nr_tag)::value;
+            const uint32_t cnt = (uint32_t)run_cnt;
+#pragma unroll 2
+            for (int j = 0; j < L; ++j) {
+                int mx = INT_MIN;
+                unsigned mn = 0xffffffffu;
+#pragma unroll
+                for (int r = 0; r < NR; ++r) {
+                    const int a = sa[r] + 1;
+                    sa[r] = a;
+                    mx = max(mx, a);
+                    mn = min(mn, (unsigned)a);
+                }
+                mx = __reduce_max_sync(kFull, mx);
+                mn = __reduce_min_sync(kFull, mn);
+                const int ext = mx - (int)mn;
+                mad_wide(W, cnt, (uint32_t)mx);      // |S| max r
+                mad_wide(sumext, (uint32_t)ext, 1u);
+                maxext = max(maxext, ext);
+                viol += ext > alpha32;
+            }
+        };
+
         // release every request with A_i <= k (a prefix: arrivals are non-decreasing)
         if (!EPOCH) {
             // ---------------------------------------------------- step kernel
             int32_t next_check = 0;   // the next step needing release / admission / the guard
-            unsigned idle_slots = 0u; // idle slots inside the used rows
             for (;;) {
                 if (k >= next_check) {
                     if (k >= step_guard) { status = ISJL_ERR_STEP_LIMIT; break; }
@@ -595,43 +682,34 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     next_check = next_arr;
                     if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) next_check = min(next_check, t0 + d1);
                     next_check = min(next_check, step_guard);
-                    idle_slots = (unsigned)(SPL * 32 - run_cnt);
                 }
-                if (run_cnt > 0) {
-                    // advance every running request by one token: r_i = a_i + 1
-                    // (all rows straight-line; idle slots advance their sentinel)
-                    int mx = INT_MIN;
-                    unsigned mn = 0xffffffffu, sm = 0u;
-#pragma unroll
-                    for (int r = 0; r < SPL; ++r) {
-                        const int a = sa[r] + 1;
-                        sa[r] = a;
-                        mx = max(mx, a);
-                        mn = min(mn, (unsigned)a);
-                        sm += (unsigned)a;
-                    }
-                    mx = __reduce_max_sync(kFull, mx);
-                    mn = __reduce_min_sync(kFull, mn);
-                    sm = __reduce_add_sync(kFull, sm);
-                    sm -= idle_slots * (unsigned)(kIdle + k);     // idle slots each added kIdle + k
-                    const int ext = mx - (int)mn;
-                    mad_wide(W, (uint32_t)run_cnt, (uint32_t)mx); // |S| max r
-                    mad_wide(R, sm, 1u);                          // sum r (>= 0)
-                    mad_wide(sumext, (uint32_t)ext, 1u);
-                    maxext = max(maxext, ext);
-                    viol += ext > alpha32;
-                    Tb++;
-                    tok += run_cnt;
-                    kvviol += kv_over;
-                    if (k + 1 == cmin) {
-                        retire(k + 1);
-                        next_check = k + 1;
-                        idle_slots = (unsigned)(SPL * 32 - run_cnt);
-                    }
+                if (run_cnt == 0) { k = next_check; continue; }   // idle steps: nothing to serve
+                // no arrival, completion, delay expiry or guard before step e
+                const int32_t e = min(next_check, cmin);
+                const int L = e - k;
+                {
+                    auto f = [&](auto nr_tag) { plain_steps(nr_tag, L); };
+                    if (adv_rows < 1) broken = true;
+                    else dispatch_rows<SPL, 0, RowClasses<SPL>::n - 1>(adv_rows, f);
                 }
-                k++;
+                if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
+                Tb += L;
+                tok += L * run_cnt;
+                if (kv_over) kvviol += L;
+                k = e;
+                if (k == cmin) {              // requests that finished in step k - 1 leave
+                    retire(k);
+                    next_check = k;
+                }
             }
-            E = W - R;
+            // requests still running (a run stopped early) served a (a + 1) / 2 so far
+#pragma unroll
+            for (int r = 0; r < SPL; ++r)
+                if (busy >> r & 1u) {
+                    const uint32_t a = (uint32_t)sa[r];
+                    mad_wide(lane_R, (a * (a + 1u)) >> 1, 1u);
+                }
+            E = W - warp_sum64(lane_R);
         } else {
             // --------------------------------------------------- epoch kernel
             for (;;) {
