@@ -45,6 +45,8 @@ DEFAULT_WID = 3
 # per workload: (policies, fairness budgets, oracle instances per host core for
 # the CPU baseline sample: one to two seconds of oracle work per core)
 GRIDS = {
+    1: (["fcfs", "ljf", "isjl"], [0, 0, 32], 1),
+    2: (["isjl"] * 5, [0, 1, 2, 4, INF], 256),
     3: (["fcfs", "ljf", "isjl", "isjl", "isjl", "isjl", "isjl"], [0, 0, 16, 64, 256, 1024, INF], 40),
     4: (["fcfs", "ljf", "isjl", "isjl", "isjl"], [0, 0, 32, 128, 512], 400),
     5: (["fcfs", "ljf", "isjl"], [0, 0, 256], 1),
@@ -59,9 +61,9 @@ ALU_LANES_PER_SM = 128
 OPS_PER_TOKEN_ADVANCE = 5
 OPS_PER_BATCH_STEP = 6
 # DRAM bytes (read + write) per launch of the step simulation kernel on the full
-# workload: 576.7 MB measured by ncu on the first 4,096 instances, scaled by
+# workload: 455.9 MB measured by ncu on the first 4,096 instances, scaled by
 # 10,000 / 4,096 (profiles/sim_kernel_step_online_delta_sweep_4096.md)
-SIM_DRAM_BYTES_PER_LAUNCH = 576.7e6 * 10_000 / 4_096
+SIM_DRAM_BYTES_PER_LAUNCH = 455.9e6 * 10_000 / 4_096
 
 
 def workload_config(kernel, wl, n_inst, policies, deltas, flush):
@@ -156,8 +158,15 @@ def host_inputs(wid, count, replica=0):
 
 def cpu_model():
     try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
         for line in open("/proc/cpuinfo"):
-            if line.lower().startswith(("model name", "cpu part")):
+            if line.lower().startswith("model name"):
                 return line.split(":", 1)[1].strip()
     except OSError:
         pass
@@ -192,7 +201,7 @@ def reference_arm(args):
     wl = W.WORKLOADS[args.workload]
     policies, deltas, per_core = GRIDS[args.workload]
     per_core = max(1, per_core * 3 // 10)
-    cores = os.cpu_count() or 1
+    cores = args.oracle_cores or os.cpu_count() or 1
     inputs = host_inputs(args.workload, cores * per_core)
     ctx = mp.get_context("spawn")
     with ctx.Pool(cores) as pool:
@@ -233,6 +242,7 @@ def main():
     ap.add_argument("--workload", type=int, choices=sorted(GRIDS), default=DEFAULT_WID)
     ap.add_argument("--instances", type=int, default=0, help="use only the first N instances (profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--oracle-cores", type=int, default=0, help="host processes for the oracle (default: all cores)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-epoch", action="store_true", help="skip the event-driven kernel's extra measurement")
     args = ap.parse_args()
@@ -248,7 +258,7 @@ def main():
 
     # the oracle pool starts before the first CUDA call (spawned workers)
     pool = None
-    cores = os.cpu_count() or 1
+    cores = args.oracle_cores or os.cpu_count() or 1
     if rank == 0 and not args.no_cpu_baseline:
         pool = mp.get_context("spawn").Pool(cores)
 
