@@ -133,7 +133,9 @@ typedef struct {
 /* Where results go.  records: device, n_runs * n_instances entries,
  * run-major (record run * n_instances + inst).  start / completion: device
  * or NULL, n_runs * n_instances * n_per_instance int32 each, run-major; the
- * step a request started / completed.  Output buffers are owned by the
+ * step a request started / completed, -1 for one that did not (an instance
+ * with an error status, a run stopped by max_steps, the unused slots of a
+ * ragged instance).  Output buffers are owned by the
  * caller and must stay valid until the run's work on the stream is done. */
 typedef struct {
     isjl_record *records;

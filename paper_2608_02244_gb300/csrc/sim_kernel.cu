@@ -241,12 +241,21 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     if (status == ISJL_OK && (int64_t)is.maxo > kv_cap) status = ISJL_ERR_INFEASIBLE;
     // every schedule ends by sum o + max arrival; the idle sentinel needs steps < 2^30
     if (status == ISJL_OK && is.O + (int64_t)is.maxA + 1 >= (int64_t)(1 << 30)) status = ISJL_ERR_INVALID_ARG;
+    // requests that never start / finish report -1: on an error status, in a
+    // run the caller's max_steps may stop, and in the unused slots of a ragged
+    // instance (a full run writes every other entry)
+    if (status != ISJL_OK || A.max_steps > 0 || n < n_slots) {
+        if (st_out) for (int i = lane; i < n_slots; i += 32) st_out[i] = -1;
+        if (co_out) for (int i = lane; i < n_slots; i += 32) co_out[i] = -1;
+    }
 
     // W = sum over steps of |S| max r; E = W - R, where R = sum over steps of
-    // sum r equals the sum over served requests of a (a + 1) / 2 for their
-    // progress a (one token per step from 1), so the step kernel adds it per
-    // request in lane_R (the decomposition W = Q + E of Section 5)
-    int64_t W = 0, lane_R = 0, E = 0, sumc = 0, sumext = 0, peakkv = 0;
+    // sum r equals the sum over served requests of a (a + 1) / 2 for the
+    // tokens a each received (one per step from 1): the step kernel adds
+    // o (o + 1) / 2 when a request starts and takes back the unserved part of
+    // requests still running if a run stops early (the decomposition W = Q + E
+    // of Section 5)
+    int64_t W = 0, R = 0, E = 0, sumc = 0, sumext = 0, peakkv = 0;
     int32_t Tb = 0, tok = 0, maxext = 0, viol = 0, peakb = 0, Tmake = 0, kvviol = 0;
 
     if (status == ISJL_OK && n > 0) {
@@ -300,10 +309,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (EPOCH) { lane_smin = INT_MAX; lane_smax = INT_MIN; }
 #pragma unroll
             for (int r = 0; r < SPL; ++r) {
-                if (busy >> r & 1u) {
-                    lane_cmin = min(lane_cmin, sc[r]);
-                    if (EPOCH) { lane_smin = min(lane_smin, sa[r]); lane_smax = max(lane_smax, sa[r]); }
-                }
+                lane_cmin = min(lane_cmin, sc[r]);               // idle slots hold INT_MAX
+                if (EPOCH && (busy >> r & 1u)) { lane_smin = min(lane_smin, sa[r]); lane_smax = max(lane_smax, sa[r]); }
             }
         };
         // start request e (length oe) on worker w at step k
@@ -316,6 +323,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             peakb = max(peakb, run_cnt);
             kv_over = kv_sum > kv_cap;
             if (EPOCH) { sum_st += k; smin = min(smin, k); smax = k; }
+            if (!EPOCH) mad_wide(R, ((uint32_t)oc * (uint32_t)(oc + 1)) >> 1, 1u);   // oc (oc + 1) < 2^32
             const int owner = w & 31, row = w >> 5;
             if (!EPOCH && row >= adv_rows) adv_rows = row_class<SPL>(row + 1);
             if (lane == owner) {
@@ -341,11 +349,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (f) {
                     if (EPOCH) sf += (unsigned)(sa[r] - (c - 65536));
                     sc[r] = INT_MAX;
-                    if (!EPOCH) {
-                        const uint32_t a = (uint32_t)sa[r];   // its length; a (a + 1) < 2^32
-                        mad_wide(lane_R, (a * (a + 1u)) >> 1, 1u);
-                        sa[r] = kIdle;
-                    }
+                    if (!EPOCH) sa[r] = kIdle;
                 }
             }
             // per finishing request (usually one per warp): outputs and its KV release
@@ -697,19 +701,21 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 tok += L * run_cnt;
                 if (kv_over) kvviol += L;
                 k = e;
-                if (k == cmin) {              // requests that finished in step k - 1 leave
+                if (k == cmin && k < step_guard) {   // requests that finished in step k - 1 leave
                     retire(k);
                     next_check = k;
                 }
             }
-            // requests still running (a run stopped early) served a (a + 1) / 2 so far
+            // a request still running (a run stopped early) with progress a and
+            // true length o = a + (completion - k) has served only a (a + 1) / 2
+            int64_t unserved = 0;
 #pragma unroll
             for (int r = 0; r < SPL; ++r)
                 if (busy >> r & 1u) {
-                    const uint32_t a = (uint32_t)sa[r];
-                    mad_wide(lane_R, (a * (a + 1u)) >> 1, 1u);
+                    const uint32_t a = (uint32_t)sa[r], o = a + (uint32_t)(sc[r] - k);
+                    unserved += (int64_t)((o * (o + 1u)) >> 1) - (int64_t)((a * (a + 1u)) >> 1);
                 }
-            E = W - warp_sum64(lane_R);
+            E = W - (R - warp_sum64(unserved));
         } else {
             // --------------------------------------------------- epoch kernel
             for (;;) {
@@ -723,6 +729,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 int32_t nxt = min(next_arr, cmin);
                 if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) nxt = min(nxt, t0 + d1);
                 if (nxt == INT_MAX) { status = ISJL_ERR_STEP_LIMIT; break; }   // cannot progress
+                nxt = min(nxt, step_guard);                          // serve no step past max_steps
                 if (run_cnt > 0) {
                     const int64_t L = nxt - k, s = run_cnt;
                     const int64_t m0 = (int64_t)k - smin + 1;       // max r at step k

@@ -284,6 +284,24 @@ def test_error_statuses(S, O, epoch):
     assert res["records"][0]["status"][0] == 5 and res["status"] == 5
 
 
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_step_limit_partial_records(S, O, epoch):
+    """A run stopped by max_steps reports exactly the steps 0..max_steps it
+    served, like the oracle: counters, partial W and E, the requests finished
+    by then, and -1 for requests that did not start or finish.  The guard is
+    also put one step before and at a completion step (the retire boundary)."""
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, o = W.generate(3, 4)
+    pols = ["fcfs", "ljf", "isjl", "isjl", "sjf"]
+    ds = [0, 0, 64, INF, 0]
+    full, _, co = O.run("fcfs", 256, 0, 200_000, a[:1], p[:1], o[:1])
+    c_mid = int(np.sort(co[0])[len(co[0]) // 2])
+    for ms in (1, 37, 1500, c_mid - 1, c_mid):
+        res = run_both(S, O, a, p, o, 256, pols, ds, 200_000, epoch, max_steps=ms)
+        assert (res["records"][0]["status"] == 5).all() and res["status"] == 5
+        assert (res["start"] == -1).any() and (res["completion"] == -1).any()
+
+
 def test_invalid_arguments_rejected(S):
     import torch
     sm = S.Simulator(1, 4, 2)
