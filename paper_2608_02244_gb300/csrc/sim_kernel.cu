@@ -210,18 +210,17 @@ __device__ __forceinline__ int first_pos_le(const int32_t *os, int n, int64_t x)
     return lo;
 }
 
-template <int SPL, bool EPOCH>
+// One (instance, run) task under policy P, a compile-time constant (FCFS, LJF,
+// SJF or ISJL; Algorithm "ISJL" runs the ISJL body with beta in the packing
+// thresholds), so each policy's code holds only its own admission rule.
+template <int SPL, bool EPOCH, int P>
 __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, int lane, int64_t gwarp,
-                                         int64_t task) {
-    const int64_t inst = task / A.n_runs;
-    const int run = (int)(task % A.n_runs);
+                                         int64_t inst, int run) {
     const int n_slots = A.n, B = A.B;
     const int64_t base = inst * (int64_t)n_slots;
     const InstStats is = A.inst[inst];
     const int n = is.n;                             // requests of this instance (<= n_slots)
-    const int policy_in = A.runs.policy[run];
-    // Algorithm "ISJL" runs the ISJL machinery with beta in the packing thresholds
-    const int policy = policy_in == ISJL_POLICY_ISJL_BETA ? ISJL_POLICY_ISJL : policy_in;
+    constexpr int policy = P;
     const int64_t alpha = A.runs.delta[run];
     const int64_t beta = A.runs.beta[run];
     const int64_t kv_cap = A.kv_cap;
@@ -819,7 +818,15 @@ sim_kernel(SimArgs A, int64_t n_tasks) {
         if (lane == 0) t = atomicAdd(A.task_counter, 1);
         t = __shfl_sync(kFull, t, 0);
         if ((int64_t)t >= n_tasks) break;
-        run_task<SPL, EPOCH>(A, S, lane, gwarp, t);
+        // run-major: at any time the warps of an SM mostly run one policy's code
+        const int64_t inst = t % A.n_inst;
+        const int run = (int)(t / A.n_inst);
+        switch (A.runs.policy[run]) {
+            case ISJL_POLICY_FCFS: run_task<SPL, EPOCH, ISJL_POLICY_FCFS>(A, S, lane, gwarp, inst, run); break;
+            case ISJL_POLICY_LJF:  run_task<SPL, EPOCH, ISJL_POLICY_LJF>(A, S, lane, gwarp, inst, run); break;
+            case ISJL_POLICY_SJF:  run_task<SPL, EPOCH, ISJL_POLICY_SJF>(A, S, lane, gwarp, inst, run); break;
+            default:               run_task<SPL, EPOCH, ISJL_POLICY_ISJL>(A, S, lane, gwarp, inst, run); break;
+        }
     }
 }
 
