@@ -200,14 +200,27 @@ __device__ __forceinline__ int bs_count_below(const WarpSmem &S, int words0, int
     return (int)__reduce_add_sync(kFull, (unsigned)cnt);
 }
 
-// first sorted position whose o is <= x (osorted is non-increasing); n if none
-__device__ __forceinline__ int first_pos_le(const int32_t *os, int n, int64_t x) {
-    int lo = 0, hi = n;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if ((int64_t)__ldg(os + mid) <= x) hi = mid; else lo = mid + 1;
+// first sorted position whose o is <= x (osorted is non-increasing); n if
+// none (uniform call).  A 32-way search: each round the lanes sample 32
+// evenly spaced positions of the bracket and a ballot keeps the sub-bracket
+// holding the answer, so n = 1,000 takes two dependent loads and n = 10^5
+// four, instead of a binary search's 10 and 17.
+__device__ __forceinline__ int first_pos_le(const int32_t *os, int n, int64_t x, int lane) {
+    int lo = 0, hi = n;                         // the answer lies in [lo, hi]
+    while (hi - lo > 32) {
+        const int step = (hi - lo + 31) >> 5;
+        const int idx = lo + lane * step;
+        const bool le = idx >= hi || (int64_t)__ldg(os + idx) <= x;
+        const unsigned b = __ballot_sync(kFull, le);
+        const int f = b ? __ffs(b) - 1 : 32;    // first sample at or after the answer
+        if (f == 0) return lo;
+        hi = min(hi, lo + f * step);
+        lo = lo + (f - 1) * step + 1;
     }
-    return lo;
+    const int idx = lo + lane;
+    const bool le = idx >= hi || (int64_t)__ldg(os + idx) <= x;
+    const unsigned b = __ballot_sync(kFull, le);
+    return b ? lo + __ffs(b) - 1 : lo + 32;
 }
 
 // One (instance, run) task under policy P, a compile-time constant (FCFS, LJF,
@@ -435,7 +448,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (p2 >= n) { broken = true; return; }
             if ((int64_t)osrt[p2] <= alpha) return;             // o_2 <= alpha: Phase TWO
             // M = min{B, #{o > alpha}} over Q(k)
-            const int cnt_long = bs_count_below(S, words0, first_pos_le(osrt, n, alpha), lane);
+            const int cnt_long = bs_count_below(S, words0, first_pos_le(osrt, n, alpha, lane), lane);
             const int nl = min(B, cnt_long);
             // packing budget left / pack sum per worker, in shared memory
             for (int w = lane; w < B; w += 32) {
@@ -474,7 +487,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 const int64_t x = min(theta, (int64_t)maxrem);
                 if (x < 1) break;
                 // candidates with o > x fit nowhere now or later (budgets only shrink)
-                q = bs_next(S, words0, words1, max(first_pos_le(osrt, n, x), q + 1), lane);
+                q = bs_next(S, words0, words1, max(first_pos_le(osrt, n, x, lane), q + 1), lane);
                 if (q >= n) break;
                 const int e = perm[q];
                 const int oe = osrt[q];
@@ -555,7 +568,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     const int hi = bs_last(S, words1, lane);
                     if (hi < 0 || hi >= n) { broken = true; return; }
                     const int omin = osrt[hi];
-                    const int p = bs_next(S, words0, words1, first_pos_le(osrt, n, omin), lane);
+                    const int p = bs_next(S, words0, words1, first_pos_le(osrt, n, omin, lane), lane);
                     if (p >= n) { broken = true; return; }
                     if (kv_sum + omin > kv_cap) break;
                     const int w = lowest_worker(vmask & ~busy, lane);
