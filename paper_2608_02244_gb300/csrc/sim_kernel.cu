@@ -191,6 +191,17 @@ __device__ __forceinline__ int bs_last(const WarpSmem &S, int words1, int lane) 
     return -1;
 }
 
+// position of the k-th (0-based) set bit of x; k < popc(x)
+__device__ __forceinline__ int nth_set_bit(uint32_t x, int k) {
+    int pos = 0;
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) {
+        const int c = __popc(x & ((1u << s) - 1u));
+        if (k >= c) { k -= c; x >>= s; pos += s; }
+    }
+    return pos;
+}
+
 // number of pending positions < P (uniform call)
 __device__ __forceinline__ int bs_count_below(const WarpSmem &S, int words0, int P, int lane) {
     const int full = P >> 5;
@@ -293,6 +304,9 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         // step kernel: register rows [0, adv_rows) are advanced each step; every
         // running worker lies in them, and their idle slots hold the sentinel
         int adv_rows = 0;
+        // step kernel: A_max at the current step, from the last step's max reduction
+        int32_t amax_c = 0;
+        bool amax_ok = false;
         int64_t kv_sum = 0, sum_st = 0;
         // the next 32 unreleased requests (from win_base): arrival and sorted position, per lane
         int32_t win_base = 0, win_a = INT_MAX, win_p = 0;
@@ -338,6 +352,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (!EPOCH) mad_wide(R, ((uint32_t)oc * (uint32_t)(oc + 1)) >> 1, 1u);   // oc (oc + 1) < 2^32
             const int owner = w & 31, row = w >> 5;
             if (!EPOCH && row >= adv_rows) adv_rows = row_class<SPL>(row + 1);
+            if (!EPOCH && run_cnt == 1) { amax_c = 0; amax_ok = true; }   // the only request: progress 0
             if (lane == owner) {
 #pragma unroll
                 for (int r = 0; r < SPL; ++r)
@@ -381,6 +396,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 sum_st -= (int64_t)__reduce_add_sync(kFull, sf) + (int64_t)nf * (c - 65536);
             done += nf;
             run_cnt -= nf;
+            if (!EPOCH && nf > 0) amax_ok = false;
             kv_sum -= of;
             kv_over = kv_sum > kv_cap;
             sumc += (int64_t)nf * c;
@@ -395,10 +411,14 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         auto amax_now = [&]() -> int64_t {
             if (run_cnt == 0) return 0;
             if (EPOCH) return (int64_t)k - smin;
-            int m = 0;
+            if (!amax_ok) {
+                int m = 0;
 #pragma unroll
-            for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = max(m, sa[r]);
-            return (int64_t)__reduce_max_sync(kFull, m);
+                for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = max(m, sa[r]);
+                amax_c = __reduce_max_sync(kFull, m);
+                amax_ok = true;
+            }
+            return amax_c;
         };
 
         auto release = [&]() {
@@ -456,26 +476,57 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 S.spsum[w] = 0;
             }
             __syncwarp();
-            // the long requests o_1..o_M leave Q; worker j's budget cap_j
-            int p = -1;
-            int64_t o_last = o1;
-            for (int j = 0; j < nl; ++j) {
-                p = bs_next(S, words0, words1, p + 1, lane);
-                if (p >= n) { broken = true; return; }
-                const int e = perm[p];
-                const int64_t oe = osrt[p];
-                bs_clear(S, p, lane);
-                if (j == 0) {
-                    L1 = e;
-                    if (lane == 0) { S.shead[0] = e; S.stail[0] = e; pnext[e] = kNone; }
-                } else {
-                    const int64_t cap = min(2 * alpha, o1 - oe + beta);
-                    if (lane == 0) S.slong[j] = e;
-                    if (lane == 0) S.srem[j] = (int32_t)cap;
+            // the long requests o_1..o_M (the first M pending positions) leave Q;
+            // worker j's budget cap_j.  Up to 32 at a time: a prefix sum of the
+            // bitset words' popcounts gives each lane the word and bit of its rank
+            int olast_l = 0;
+            for (int wb = 0, taken = 0; taken < nl; wb += 32) {
+                if (wb >= words0) { broken = true; return; }
+                const int wi = wb + lane;
+                const uint32_t x = wi < words0 ? S.pend0[wi] : 0u;
+                const int c = __popc(x);
+                int incl = c;                                   // inclusive count over lanes
+#pragma unroll
+                for (int d = 1; d < 32; d <<= 1) {
+                    const int t = __shfl_up_sync(kFull, incl, d);
+                    if (lane >= d) incl += t;
                 }
-                o_last = oe;
+                const int excl = incl - c;
+                const int m = min(nl - taken, __shfl_sync(kFull, incl, 31));   // ranks from this chunk
+                for (int r0 = 0; r0 < m; r0 += 32) {
+                    const int jj = r0 + lane;                       // rank within the chunk
+                    int lo = 0;                                     // lanes whose words end before it
+#pragma unroll
+                    for (int sh = 16; sh > 0; sh >>= 1)
+                        if (__shfl_sync(kFull, incl, lo + sh - 1) <= jj) lo += sh;
+                    const uint32_t xw = __shfl_sync(kFull, x, lo);
+                    const int ew = __shfl_sync(kFull, excl, lo);
+                    if (jj < m) {
+                        const int p = ((wb + lo) << 5) + nth_set_bit(xw, jj - ew);
+                        const int j = taken + jj;
+                        const int e = perm[p];
+                        const int oe = osrt[p];
+                        if (j == 0) {
+                            S.shead[0] = e; S.stail[0] = e; pnext[e] = kNone;
+                        } else {
+                            S.slong[j] = e;
+                            S.srem[j] = (int32_t)min(2 * alpha, o1 - (int64_t)oe + beta);
+                        }
+                        if (j == nl - 1) olast_l = oe;
+                    }
+                }
+                // the taken bits of this lane's word leave the bitset
+                const int tk = min(max(m - excl, 0), c);
+                if (tk > 0) {
+                    const uint32_t y = tk == c ? 0u : x & (~0u << nth_set_bit(x, tk));
+                    S.pend0[wi] = y;
+                    if (y == 0u) atomicAnd(&S.pend1[wi >> 5], ~(1u << (wi & 31)));
+                }
+                taken += m;
             }
             __syncwarp();
+            L1 = S.shead[0];
+            const int64_t o_last = __reduce_max_sync(kFull, olast_l);
             pend -= nl;
             const int64_t theta = min(2 * alpha, o1 - o_last + beta);
             // first fit of the shorter requests, in sorted order
@@ -663,6 +714,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         auto plain_steps = [&](auto nr_tag, int L) {
             constexpr int NR = decltype(nr_tag)::value;
             const uint32_t cnt = (uint32_t)run_cnt;
+            int last_mx = 0;
 #pragma unroll 2
             for (int j = 0; j < L; ++j) {
                 int mx = INT_MIN;
@@ -681,7 +733,10 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 mad_wide(sumext, (uint32_t)ext, 1u);
                 maxext = max(maxext, ext);
                 viol += ext > alpha32;
+                last_mx = mx;
             }
+            amax_c = last_mx;                        // max progress entering step k + L
+            amax_ok = true;
         };
 
         // release every request with A_i <= k (a prefix: arrivals are non-decreasing)
