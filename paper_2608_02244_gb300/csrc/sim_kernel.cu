@@ -601,12 +601,24 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             __syncwarp();
         };
 
+        // After an admission, `blocked` says that no arrival alone can let a
+        // request start before the next completion (or o_1's delay expiry):
+        // FCFS with B full or its head not fitting the KV cap, LJF with a batch
+        // running, SJF with B full, ISJL with its gate closed or its queue
+        // stopped on the KV cap or on workers (an arrival never becomes a head
+        // that fits better: it sorts after every pending request of its length).
+        // Arrivals are then released at the next event instead of ending the
+        // run of plain steps there.
+        bool blocked = false;
         auto admit = [&]() {
             if (policy == ISJL_POLICY_FCFS) {
                 // arrival order; the first request that does not fit ends the step
-                while (run_cnt < B && fcfs < rel) {
+                blocked = false;
+                for (;;) {
+                    if (run_cnt >= B) { blocked = true; break; }
+                    if (fcfs >= rel) break;
                     if (fo < 0) fo = oarr[fcfs];
-                    if (kv_sum + fo > kv_cap) break;
+                    if (kv_sum + fo > kv_cap) { blocked = true; break; }
                     const int w = lowest_worker(vmask & ~busy, lane);
                     if (w < 0) { broken = true; return; }
                     start(fcfs, fo, w);
@@ -629,8 +641,10 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     pend--;
                     start(e, omin, w);
                 }
+                blocked = run_cnt >= B;
             } else if (policy == ISJL_POLICY_LJF) {
                 // static batch of the longest released requests when nothing runs
+                blocked = run_cnt != 0;
                 if (run_cnt != 0) return;
                 while (run_cnt < B && pend > 0) {
                     const int p = head();
@@ -643,6 +657,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     pop_head(p);
                     start(e, oe, w);
                 }
+                blocked = run_cnt != 0;
             } else {
                 const bool nothing_runs = run_cnt == 0;
                 if (nothing_runs && plan_left == 0 && pend > 0) phase_one();
@@ -704,6 +719,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         start(e, oe, w);
                     }
                 }
+                blocked = stop || pend > 0;
             }
         };
 
@@ -750,7 +766,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     if (k >= next_arr) release();
                     admit();
                     if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
-                    next_check = next_arr;
+                    next_check = blocked && run_cnt > 0 ? INT_MAX : next_arr;
                     if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) next_check = min(next_check, t0 + d1);
                     next_check = min(next_check, step_guard);
                 }
@@ -793,7 +809,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 admit();
                 if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
                 // next event: arrival, completion or the end of o_1's delay
-                int32_t nxt = min(next_arr, cmin);
+                int32_t nxt = min(blocked && run_cnt > 0 ? INT_MAX : next_arr, cmin);
                 if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) nxt = min(nxt, t0 + d1);
                 if (nxt == INT_MAX) { status = ISJL_ERR_STEP_LIMIT; break; }   // cannot progress
                 nxt = min(nxt, step_guard);                          // serve no step past max_steps
