@@ -318,7 +318,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         load_window();
         // uniform caches, changed only at events
         int32_t next_arr = __shfl_sync(kFull, win_a, 0);   // arrival of the next unreleased request
-        int32_t hp = INT_MAX, ho = 0, ho_pos = -1;     // longest pending position and its o (LJF / ISJL)
+        int32_t hp = INT_MAX, ho = 0, he = 0, ho_pos = -1;   // longest pending position, its o and index
         bool hvalid = true;                            // hp is current (else recompute from the bitset)
         int32_t fo = -1;                               // o of the FCFS head (-1: not loaded)
         int32_t cmin = INT_MAX;                        // earliest completion step of the running set
@@ -364,6 +364,74 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 S.sjob[w] = e;
                 if (st_out) st_out[e] = k;
             }
+        };
+        // Start, at step k, the longest prefix of up to 32 candidates (lane l < m
+        // holds request ce and its planning length co) whose KV reservations fit
+        // and for which free workers remain, candidate i on the i-th lowest
+        // worker of the free mask fm.  The same outcome as starting them one at
+        // a time, each on the lowest free worker, until the first that does not
+        // fit.  Returns how many started.
+        auto bulk_start = [&](int m, int ce, int co, uint32_t fm) -> int {
+            int pre = lane < m ? co : 0;                          // inclusive prefix of co
+#pragma unroll
+            for (int d = 1; d < 32; d <<= 1) {
+                const int t = __shfl_up_sync(kFull, pre, d);
+                if (lane >= d) pre += t;
+            }
+            const int nfree = (int)__reduce_add_sync(kFull, (unsigned)__popc(fm));
+            const bool fit = lane < m && lane < nfree && kv_sum + pre <= kv_cap;
+            const int c = __popc(__ballot_sync(kFull, fit));
+            if (c == 0) return 0;
+            const int oc_l = (otru && lane < c) ? otru[ce] : co;  // it finishes after its true length
+            const uint32_t lt = (1u << lane) - 1u;
+            int base = 0, top = 0;
+            int32_t my_cmin = INT_MAX;
+            uint64_t rsum = 0;
+#pragma unroll
+            for (int r = 0; r < SPL; ++r) {
+                if (base < c) {
+                    const bool f = fm >> r & 1u;
+                    const unsigned rowf = __ballot_sync(kFull, f);
+                    const int rank = base + __popc(rowf & lt);     // among the free workers, in w order
+                    const int src = rank & 31;
+                    const int e = __shfl_sync(kFull, ce, src);
+                    const int oe = __shfl_sync(kFull, co, src);
+                    const int oc = __shfl_sync(kFull, oc_l, src);
+                    if (f && rank < c) {
+                        const int w = (r << 5) + lane;
+                        sa[r] = EPOCH ? k : 0;
+                        sc[r] = k + oc;
+                        busy |= 1u << r;
+                        my_cmin = min(my_cmin, k + oc);
+                        S.sres[w] = oe;
+                        S.sjob[w] = e;
+                        if (st_out) st_out[e] = k;
+                        if (!EPOCH) rsum += ((uint32_t)oc * (uint32_t)(oc + 1)) >> 1;
+                    }
+                    if (rowf) top = r + 1;
+                    base += __popc(rowf);
+                }
+            }
+            __syncwarp();
+            lane_cmin = min(lane_cmin, my_cmin);
+            if (EPOCH && my_cmin != INT_MAX) { lane_smin = min(lane_smin, k); lane_smax = max(lane_smax, k); }
+            const bool was_empty = run_cnt == 0;
+            run_cnt += c;
+            kv_sum += __shfl_sync(kFull, pre, c - 1);
+            cmin = min(cmin, (int32_t)__reduce_min_sync(kFull, (unsigned)my_cmin));
+            peakkv = max(peakkv, kv_sum);
+            peakb = max(peakb, run_cnt);
+            kv_over = kv_sum > kv_cap;
+            if (EPOCH) { sum_st += (int64_t)c * k; smin = min(smin, k); smax = k; }
+            if (!EPOCH) {
+                // rsum < 2^35 per lane: its low 24 bits and the rest summed by two reductions
+                const unsigned lo = __reduce_add_sync(kFull, (unsigned)(rsum & 0xFFFFFFu));
+                const unsigned hi = __reduce_add_sync(kFull, (unsigned)(rsum >> 24));
+                R += ((int64_t)hi << 24) + (int64_t)lo;
+                if (top > adv_rows) adv_rows = row_class<SPL>(top);
+                if (was_empty) { amax_c = 0; amax_ok = true; }   // the new requests: progress 0
+            }
+            return c;
         };
         // requests completing at step c leave their workers
         auto retire = [&](int32_t c) {
@@ -443,10 +511,10 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             __syncwarp();
             next_arr = rel < n ? __shfl_sync(kFull, win_a, (rel - win_base) & 31) : INT_MAX;
         };
-        // longest pending position (INT_MAX if none) and its length
+        // longest pending position (INT_MAX if none), its o and request index
         auto head = [&]() -> int {
             if (!hvalid) { hp = bs_next(S, words0, words1, 0, lane); hvalid = true; }
-            if (hp < n && ho_pos != hp) { ho = osrt[hp]; ho_pos = hp; }
+            if (hp < n && ho_pos != hp) { ho = osrt[hp]; he = perm[hp]; ho_pos = hp; }
             return hp;
         };
         // remove the head position p (the longest pending request)
@@ -454,6 +522,76 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             bs_clear(S, p, lane);
             pend--;
             hp = bs_next(S, words0, words1, p + 1, lane);   // nothing pending below p
+        };
+        // sorted positions of the first m (1 <= m <= min(32, pend)) pending
+        // requests: lane l < m gets the l-th, the other lanes -1 (uniform call)
+        auto first_pending = [&](int m) -> int {
+            int mine = -1;
+            if (!hvalid) { hp = bs_next(S, words0, words1, 0, lane); hvalid = true; }
+            const int p0 = hp;
+            for (int wb = (p0 >> 10) << 5, got = 0; got < m && wb < words0; wb += 32) {
+                if (S.pend1[wb >> 5] == 0u) continue;           // no pending in these 32 words
+                const int wi = wb + lane;
+                const uint32_t x = wi < words0 ? S.pend0[wi] : 0u;
+                const int c = __popc(x);
+                int incl = c;
+#pragma unroll
+                for (int d = 1; d < 32; d <<= 1) {
+                    const int t = __shfl_up_sync(kFull, incl, d);
+                    if (lane >= d) incl += t;
+                }
+                const int excl = incl - c;
+                const int jj = lane - got;                      // this lane's rank within the chunk
+                int lo = 0;
+#pragma unroll
+                for (int sh = 16; sh > 0; sh >>= 1)
+                    if (__shfl_sync(kFull, incl, lo + sh - 1) <= jj) lo += sh;
+                const uint32_t xw = __shfl_sync(kFull, x, lo);
+                const int ew = __shfl_sync(kFull, excl, lo);
+                const int tot = __shfl_sync(kFull, incl, 31);
+                if (lane < m && jj >= 0 && jj < tot) mine = ((wb + lo) << 5) + nth_set_bit(xw, jj - ew);
+                got += tot;
+            }
+            return mine;
+        };
+        // remove the lanes' positions p (where take) from the pending set
+        auto clear_pending = [&](int p, bool take) {
+            if (take) {
+                const uint32_t bit = 1u << (p & 31);
+                const uint32_t old = atomicAnd(&S.pend0[p >> 5], ~bit);
+                if ((old & ~bit) == 0u) atomicAnd(&S.pend1[p >> 10], ~(1u << ((p >> 5) & 31)));
+            }
+            __syncwarp();
+        };
+        // start the longest pending requests (LJF's batch, ISJL's Phase TWO) on
+        // the free workers of fm_base until one does not fit or the workers run out
+        auto start_longest = [&](uint32_t fm_base) -> void {
+            // one at a time for the first two starts (usually all there are),
+            // then 32 at a time; every round first checks that the head fits
+            for (int nseq = 0; pend > 0;) {
+                const int w = lowest_worker(fm_base & ~busy, lane);
+                if (w < 0) return;
+                const int p = head();
+                if (p >= n) { broken = true; return; }
+                if (kv_sum + ho > kv_cap) return;
+                if (nseq < 2) {
+                    const int e = he, oe = ho;
+                    pop_head(p);
+                    start(e, oe, w);
+                    nseq++;
+                    continue;
+                }
+                const int m = min(32, pend);
+                const int q = first_pending(m);
+                if (__ballot_sync(kFull, lane < m && q < 0)) { broken = true; return; }
+                const int ce = q >= 0 ? perm[q] : 0;
+                const int co = q >= 0 ? osrt[q] : 0;
+                const int c = bulk_start(m, ce, co, fm_base & ~busy);
+                clear_pending(q, lane < c);
+                pend -= c;
+                if (c < m) { hp = __shfl_sync(kFull, q, c); return; }   // the first one left is the head
+                hvalid = false;
+            }
         };
 
         // ISJL Phase ONE at a stage start (Algorithm 2 with beta = alpha)
@@ -614,16 +752,28 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (policy == ISJL_POLICY_FCFS) {
                 // arrival order; the first request that does not fit ends the step
                 blocked = false;
-                for (;;) {
+                // one at a time for the first two starts (usually all there are),
+                // then 32 at a time; every round first checks that the head fits
+                for (int nseq = 0;;) {
                     if (run_cnt >= B) { blocked = true; break; }
                     if (fcfs >= rel) break;
                     if (fo < 0) fo = oarr[fcfs];
                     if (kv_sum + fo > kv_cap) { blocked = true; break; }
-                    const int w = lowest_worker(vmask & ~busy, lane);
-                    if (w < 0) { broken = true; return; }
-                    start(fcfs, fo, w);
-                    fcfs++;
+                    if (nseq < 2) {
+                        const int w = lowest_worker(vmask & ~busy, lane);
+                        if (w < 0) { broken = true; return; }
+                        start(fcfs, fo, w);
+                        fcfs++;
+                        fo = -1;
+                        nseq++;
+                        continue;
+                    }
+                    const int m = min(32, rel - fcfs);
+                    const int i = fcfs + lane;
+                    const int c = bulk_start(m, i, lane < m ? oarr[i] : 0, vmask & ~busy);
+                    fcfs += c;
                     fo = -1;
+                    if (c < m) { blocked = true; break; }        // the KV cap or B stopped it
                 }
             } else if (policy == ISJL_POLICY_SJF) {
                 // shortest released request first (ties: lower index), continuous batching
@@ -646,17 +796,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 // static batch of the longest released requests when nothing runs
                 blocked = run_cnt != 0;
                 if (run_cnt != 0) return;
-                while (run_cnt < B && pend > 0) {
-                    const int p = head();
-                    if (p >= n) { broken = true; return; }
-                    if (kv_sum + ho > kv_cap) break;
-                    const int e = perm[p];
-                    const int w = lowest_worker(vmask & ~busy, lane);
-                    if (w < 0) { broken = true; return; }
-                    const int oe = ho;
-                    pop_head(p);
-                    start(e, oe, w);
-                }
+                start_longest(vmask);
                 blocked = run_cnt != 0;
             } else {
                 const bool nothing_runs = run_cnt == 0;
@@ -705,20 +845,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         start(e, oe, w);
                     }
                 }
-                if (!stop) {
-                    // Phase TWO: longest released request onto a free worker
-                    while (pend > 0) {
-                        const int w = lowest_worker(vmask & ~busy & ~resv, lane);
-                        if (w < 0) break;
-                        const int p = head();
-                        if (p >= n) { broken = true; return; }
-                        if (kv_sum + ho > kv_cap) break;
-                        const int e = perm[p];
-                        const int oe = ho;
-                        pop_head(p);
-                        start(e, oe, w);
-                    }
-                }
+                if (!stop) start_longest(vmask & ~resv);   // Phase TWO: longest released first
                 blocked = stop || pend > 0;
             }
         };
