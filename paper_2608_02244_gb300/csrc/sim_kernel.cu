@@ -80,7 +80,7 @@ template <int N> struct RowCount { static constexpr int value = N; };
 // Row counts the step loop is instantiated for, per SPL (ascending).  The
 // loop advances the smallest of them covering every running worker; a few
 // classes keep the kernel small (measured: powers of two for SPL = 8, even
-// counts for SPL = 16), and its steps are unrolled by two.
+// counts for SPL = 16), and its steps are unrolled by four.
 template <int SPL> struct RowClasses;
 template <> struct RowClasses<1> {
     static constexpr int n = 1;
@@ -858,7 +858,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             constexpr int NR = decltype(nr_tag)::value;
             const uint32_t cnt = (uint32_t)run_cnt;
             int last_mx = 0;
-#pragma unroll 2
+#pragma unroll 4
             for (int j = 0; j < L; ++j) {
                 int mx = INT_MIN;
                 unsigned mn = 0xffffffffu;
