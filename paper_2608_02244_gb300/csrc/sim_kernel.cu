@@ -365,6 +365,30 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (st_out) st_out[e] = k;
             }
         };
+        // warp-wide totals of c starts at step k made lane-parallel: kv_add their
+        // reserved KV, my_cmin / rsum this lane's earliest completion and sum of
+        // o (o + 1) / 2, top the highest row that received one, plus one
+        auto commit_starts = [&](int c, int64_t kv_add, int32_t my_cmin, uint64_t rsum, int top) {
+            __syncwarp();
+            lane_cmin = min(lane_cmin, my_cmin);
+            if (EPOCH && my_cmin != INT_MAX) { lane_smin = min(lane_smin, k); lane_smax = max(lane_smax, k); }
+            const bool was_empty = run_cnt == 0;
+            run_cnt += c;
+            kv_sum += kv_add;
+            cmin = min(cmin, (int32_t)__reduce_min_sync(kFull, (unsigned)my_cmin));
+            peakkv = max(peakkv, kv_sum);
+            peakb = max(peakb, run_cnt);
+            kv_over = kv_sum > kv_cap;
+            if (EPOCH) { sum_st += (int64_t)c * k; smin = min(smin, k); smax = k; }
+            if (!EPOCH) {
+                // rsum < 2^35 per lane: its low 24 bits and the rest summed by two reductions
+                const unsigned lo = __reduce_add_sync(kFull, (unsigned)(rsum & 0xFFFFFFu));
+                const unsigned hi = __reduce_add_sync(kFull, (unsigned)(rsum >> 24));
+                R += ((int64_t)hi << 24) + (int64_t)lo;
+                if (top > adv_rows) adv_rows = row_class<SPL>(top);
+                if (was_empty) { amax_c = 0; amax_ok = true; }   // the new requests: progress 0
+            }
+        };
         // Start, at step k, the longest prefix of up to 32 candidates (lane l < m
         // holds request ce and its planning length co) whose KV reservations fit
         // and for which free workers remain, candidate i on the i-th lowest
@@ -412,25 +436,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     base += __popc(rowf);
                 }
             }
-            __syncwarp();
-            lane_cmin = min(lane_cmin, my_cmin);
-            if (EPOCH && my_cmin != INT_MAX) { lane_smin = min(lane_smin, k); lane_smax = max(lane_smax, k); }
-            const bool was_empty = run_cnt == 0;
-            run_cnt += c;
-            kv_sum += __shfl_sync(kFull, pre, c - 1);
-            cmin = min(cmin, (int32_t)__reduce_min_sync(kFull, (unsigned)my_cmin));
-            peakkv = max(peakkv, kv_sum);
-            peakb = max(peakb, run_cnt);
-            kv_over = kv_sum > kv_cap;
-            if (EPOCH) { sum_st += (int64_t)c * k; smin = min(smin, k); smax = k; }
-            if (!EPOCH) {
-                // rsum < 2^35 per lane: its low 24 bits and the rest summed by two reductions
-                const unsigned lo = __reduce_add_sync(kFull, (unsigned)(rsum & 0xFFFFFFu));
-                const unsigned hi = __reduce_add_sync(kFull, (unsigned)(rsum >> 24));
-                R += ((int64_t)hi << 24) + (int64_t)lo;
-                if (top > adv_rows) adv_rows = row_class<SPL>(top);
-                if (was_empty) { amax_c = 0; amax_ok = true; }   // the new requests: progress 0
-            }
+            commit_starts(c, __shfl_sync(kFull, pre, c - 1), my_cmin, rsum, top);
             return c;
         };
         // requests completing at step c leave their workers
@@ -592,6 +598,67 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (c < m) { hp = __shfl_sync(kFull, q, c); return; }   // the first one left is the head
                 hvalid = false;
             }
+        };
+
+        // ISJL plan starts of every candidate worker in cand (per-lane row
+        // mask) at once, in worker order, until the first whose next entry does
+        // not fit the KV cap (then true is returned: the gate of the step is
+        // shut); entries that must wait (o_1 delayed unless over, an o_j before
+        // o_1 has started) are skipped.  o_1 itself never comes here: worker 0
+        // is always the first candidate and is started one at a time.
+        auto plan_bulk = [&](uint32_t cand, bool over) -> bool {
+            bool stopped = false;
+            int c = 0, top = 0;
+            int64_t kv_add = 0;
+            int32_t my_cmin = INT_MAX;
+            uint64_t rsum = 0;
+#pragma unroll
+            for (int r = 0; r < SPL; ++r) {
+                if (!stopped) {
+                    const int w = (r << 5) + lane;
+                    bool el = cand >> r & 1u;
+                    int e = 0, oe = 0;
+                    if (el) {
+                        e = S.shead[w];
+                        if (w == 0 && e == L1 && !over) el = false;
+                        if (w >= 1 && w < nlong && e == S.slong[w] && !L1_started) el = false;
+                        if (el) oe = S.spsum[w];
+                    }
+                    int pre = el ? oe : 0;                      // prefix over this row, in lane order
+#pragma unroll
+                    for (int d = 1; d < 32; d <<= 1) {
+                        const int t = __shfl_up_sync(kFull, pre, d);
+                        if (lane >= d) pre += t;
+                    }
+                    const bool fits = el && kv_sum + kv_add + pre <= kv_cap;
+                    const unsigned fb = __ballot_sync(kFull, fits);
+                    if (fb != __ballot_sync(kFull, el)) stopped = true;   // the first one that does not fit
+                    if (fits) {
+                        const int nx = pnext[e];
+                        const int onx = nx >= 0 ? oarr[nx] : 0;
+                        S.shead[w] = nx;
+                        const uint32_t bit = 1u << r;
+                        if (nx < 0) { S.stail[w] = kNone; resv &= ~bit; } else S.spsum[w] = onx;
+                        if (w >= 1 && w < nlong && nx >= 0 && nx == S.slong[w]) lhead |= bit;
+                        else lhead &= ~bit;
+                        const int oc = otru ? otru[e] : oe;     // it finishes after its true length
+                        sa[r] = EPOCH ? k : 0;
+                        sc[r] = k + oc;
+                        busy |= bit;
+                        my_cmin = min(my_cmin, k + oc);
+                        S.sres[w] = oe;
+                        S.sjob[w] = e;
+                        if (st_out) st_out[e] = k;
+                        if (!EPOCH) rsum += ((uint32_t)oc * (uint32_t)(oc + 1)) >> 1;
+                    }
+                    if (fb) top = r + 1;
+                    c += __popc(fb);
+                    kv_add += (int64_t)__reduce_add_sync(kFull, fits ? (unsigned)oe : 0u);
+                }
+            }
+            if (c > 0) commit_starts(c, kv_add, my_cmin, rsum, top);
+            plan_left -= c;
+            return stopped;
         };
 
         // ISJL Phase ONE at a stage start (Algorithm 2 with beta = alpha)
@@ -812,7 +879,14 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         const bool over = ((int64_t)k >= (int64_t)t0 + d1) || (k > t0 && nothing_runs);
                         if (!over && lane == 0) cand &= ~1u;        // worker 0 holds o_1
                     }
-                    for (;;) {
+                    for (int nseq = 0;;) {
+                        if (nseq >= 2) {                            // the rest at once
+                            if (__ballot_sync(kFull, cand != 0u)) {
+                                const bool over = ((int64_t)k >= (int64_t)t0 + d1) || (k > t0 && nothing_runs);
+                                stop = plan_bulk(cand, over);
+                            }
+                            break;
+                        }
                         const int w = lowest_worker(cand, lane);
                         if (w < 0) break;
                         if (lane == (w & 31)) cand &= ~(1u << (w >> 5));
@@ -843,6 +917,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                             cand |= resv & ~busy & lhead;            // the o_j may start now
                         }
                         start(e, oe, w);
+                        nseq++;
                     }
                 }
                 if (!stop) start_longest(vmask & ~resv);   // Phase TWO: longest released first
