@@ -345,23 +345,29 @@ def main():
                  "ms_per_step": sum(step2) / args.steps, "sim_ms_per_launch": sum(sim2) / len(sim2)}
         S2.close()
 
-    # e2e through the host-memory entry point: H2D of the inputs, sweep, D2H of
-    # the records (that entry point takes no counts or slack arrays)
+    # e2e through the host-memory entry point: H2D of the inputs (and counts /
+    # slack where the workload has them), sweep, D2H of the records
     e2e = None
-    if not args.no_e2e and c_h is None and e_h is None:
+    if not args.no_e2e:
         pa, pp, po = (torch.from_numpy(x).pin_memory() for x in (a_h, p_h, o_h))
+        pc = torch.from_numpy(c_h).pin_memory() if c_h is not None else None
+        pe = torch.from_numpy(e_h).pin_memory() if e_h is not None else None
         hrec = torch.empty(len(policies) * n_inst * sim.RECORD_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
-        sim.isjl_sim_run_sweep_host(S.handle, policies, deltas, kv, pa, pp, po, hrec)   # warm
+
+        def host_sweep():
+            return sim.isjl_sim_run_sweep_host(S.handle, policies, deltas, kv, pa, pp, po, hrec, h_count=pc,
+                                               h_slack=pe)
+        host_sweep()   # warm
         torch.cuda.synchronize()
         e2e_ms = []
         for _ in range(args.steps):
             t0 = time.perf_counter()
-            rc = sim.isjl_sim_run_sweep_host(S.handle, policies, deltas, kv, pa, pp, po, hrec)
+            rc = host_sweep()
             e2e_ms.append(1e3 * (time.perf_counter() - t0))
             if rc != 0:
                 raise RuntimeError(f"host sweep status {rc}")
-        e2e = {"ms": sum(e2e_ms) / len(e2e_ms),
-               "h2d": 3 * a_h.nbytes, "d2h": hrec.numel()}
+        h2d = 3 * a_h.nbytes + (c_h.nbytes if c_h is not None else 0) + (e_h.nbytes if e_h is not None else 0)
+        e2e = {"ms": sum(e2e_ms) / len(e2e_ms), "h2d": h2d, "d2h": hrec.numel()}
 
     # max over ranks, sum of units
     units = float(busy_per_step * args.steps)

@@ -189,15 +189,19 @@ isjl_status isjl_sim_run_sweep(isjl_sim *sim, int32_t n_runs, const int32_t *pol
                                const isjl_instances *in, const isjl_outputs *out, void *stream);
 
 /* The same sweep from and to HOST memory: copies the three input arrays
- * (n_instances * n_per_instance int32 each) to the device, simulates, and
- * copies the n_runs * n_instances records back into h_records, all on
- * stream, then synchronizes it.  The first call allocates the device input
- * and record buffers (kept until destroy).  Errors: as isjl_sim_run_sweep,
- * plus OOM on first use, plus the first device status (as isjl_sim_metrics). */
+ * (n_instances * n_per_instance int32 each) and, when not NULL, the request
+ * counts (n_instances int32, as isjl_instances.count) and the upper-bound
+ * slack (n_instances * n_per_instance int32, as isjl_instances.slack) to the
+ * device, simulates, and copies the n_runs * n_instances records back into
+ * h_records, all on stream, then synchronizes it.  The first call allocates
+ * the device input and record buffers, the first call with counts or slack
+ * their buffers (kept until destroy).  Errors: as isjl_sim_run_sweep, plus OOM
+ * on first use, plus the first device status (as isjl_sim_metrics). */
 isjl_status isjl_sim_run_sweep_host(isjl_sim *sim, int32_t n_runs, const int32_t *policies,
                                     const int32_t *deltas, int32_t kv_cap,
                                     const int32_t *h_arrival, const int32_t *h_prompt,
-                                    const int32_t *h_output, isjl_record *h_records, void *stream);
+                                    const int32_t *h_output, const int32_t *h_count,
+                                    const int32_t *h_slack, isjl_record *h_records, void *stream);
 
 /* Wait for the last run/sweep on its stream and copy its per-run summaries
  * into the host array out (capacity max_runs >= the last call's n_runs).

@@ -23,6 +23,7 @@ struct isjl_sim {
     isjl_summary *d_summary = nullptr;
     // buffers of the host-memory entry point, allocated on first use
     int32_t *d_in[3] = {nullptr, nullptr, nullptr};
+    int32_t *d_cnt_in = nullptr, *d_slack_in = nullptr;   // host-entry counts and slack
     isjl_record *d_rec_io = nullptr;
     // last call
     cudaStream_t last_stream = nullptr;
@@ -45,7 +46,8 @@ void free_all(isjl_sim *s) {
     for (cudaEvent_t &e : s->ev)
         if (e) { cudaEventDestroy(e); e = nullptr; }
     void *ptrs[] = {s->d_o, s->d_otrue, s->d_perm, s->d_osorted, s->d_posof, s->d_tmp, s->d_inst, s->d_plan_next,
-                    s->d_counter, s->d_status, s->d_summary, s->d_in[0], s->d_in[1], s->d_in[2], s->d_rec_io};
+                    s->d_counter, s->d_status, s->d_summary, s->d_in[0], s->d_in[1], s->d_in[2], s->d_rec_io,
+                    s->d_cnt_in, s->d_slack_in};
     for (void *p : ptrs)
         if (p) cudaFree(p);
 }
@@ -219,7 +221,8 @@ isjl_status isjl_sim_metrics(isjl_sim *s, isjl_summary *out, int32_t max_runs) {
 
 isjl_status isjl_sim_run_sweep_host(isjl_sim *s, int32_t n_runs, const int32_t *policies, const int32_t *deltas,
                                     int32_t kv_cap, const int32_t *h_arrival, const int32_t *h_prompt,
-                                    const int32_t *h_output, isjl_record *h_records, void *stream) {
+                                    const int32_t *h_output, const int32_t *h_count, const int32_t *h_slack,
+                                    isjl_record *h_records, void *stream) {
     if (!s || !h_arrival || !h_prompt || !h_output || !h_records || !valid_runs(n_runs, policies, deltas) ||
         kv_cap < 1)
         return ISJL_ERR_INVALID_ARG;
@@ -236,12 +239,23 @@ isjl_status isjl_sim_run_sweep_host(isjl_sim *s, int32_t n_runs, const int32_t *
             return ISJL_ERR_OOM;
         }
     }
+    if ((h_count && !s->d_cnt_in && dalloc(&s->d_cnt_in, (size_t)s->cfg.n_instances) != cudaSuccess) ||
+        (h_slack && !s->d_slack_in && dalloc(&s->d_slack_in, s->N) != cudaSuccess)) {
+        cudaGetLastError();
+        return ISJL_ERR_OOM;
+    }
     const size_t bytes = sizeof(int32_t) * (size_t)s->N;
     const int32_t *src[3] = {h_arrival, h_prompt, h_output};
     for (int i = 0; i < 3; ++i)
         if (cudaMemcpyAsync(s->d_in[i], src[i], bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
             return ISJL_ERR_CUDA;
-    isjl_instances in{s->d_in[0], s->d_in[1], s->d_in[2]};
+    if (h_count && cudaMemcpyAsync(s->d_cnt_in, h_count, sizeof(int32_t) * (size_t)s->cfg.n_instances,
+                                   cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return ISJL_ERR_CUDA;
+    if (h_slack && cudaMemcpyAsync(s->d_slack_in, h_slack, bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return ISJL_ERR_CUDA;
+    isjl_instances in{s->d_in[0], s->d_in[1], s->d_in[2], h_count ? s->d_cnt_in : nullptr,
+                      h_slack ? s->d_slack_in : nullptr};
     isjl_outputs out{s->d_rec_io, nullptr, nullptr};
     isjl_status rs = isjl_sim_run_sweep(s, n_runs, policies, deltas, kv_cap, &in, &out, stream);
     if (rs != ISJL_OK) return rs;

@@ -86,7 +86,7 @@ def lib():
         L.isjl_sim_run_sweep.argtypes = [vp, i32, p32, p32, i32, ctypes.POINTER(isjl_instances),
                                          ctypes.POINTER(isjl_outputs), vp]
         L.isjl_sim_run_sweep.restype = ctypes.c_int
-        L.isjl_sim_run_sweep_host.argtypes = [vp, i32, p32, p32, i32, vp, vp, vp, vp, vp]
+        L.isjl_sim_run_sweep_host.argtypes = [vp, i32, p32, p32, i32, vp, vp, vp, vp, vp, vp, vp]
         L.isjl_sim_run_sweep_host.restype = ctypes.c_int
         L.isjl_sim_metrics.argtypes = [vp, ctypes.POINTER(isjl_summary), i32]
         L.isjl_sim_metrics.restype = ctypes.c_int
@@ -176,14 +176,17 @@ def isjl_sim_run_sweep(handle, policies, deltas, kv_cap, arrival, prompt, output
 
 
 def isjl_sim_run_sweep_host(handle, policies, deltas, kv_cap, h_arrival, h_prompt, h_output, h_records,
-                            stream=None):
-    """Host-memory sweep: h_* are pinned (or pageable) torch CPU int32 tensors,
-    h_records a CPU uint8 tensor of n_runs * n_instances * 192 bytes."""
+                            stream=None, h_count=None, h_slack=None):
+    """Host-memory sweep: h_* are pinned (or pageable) torch CPU int32 tensors
+    (h_count / h_slack optional), h_records a CPU uint8 tensor of
+    n_runs * n_instances * 192 bytes."""
     pol = _i32_array([_policy_code(p) for p in policies])
     dl = _i32_array(deltas)
     return lib().isjl_sim_run_sweep_host(handle, len(pol), pol, dl, int(kv_cap), h_arrival.data_ptr(),
-                                         h_prompt.data_ptr(), h_output.data_ptr(), h_records.data_ptr(),
-                                         _stream_ptr(stream))
+                                         h_prompt.data_ptr(), h_output.data_ptr(),
+                                         h_count.data_ptr() if h_count is not None else None,
+                                         h_slack.data_ptr() if h_slack is not None else None,
+                                         h_records.data_ptr(), _stream_ptr(stream))
 
 
 def isjl_sim_run_sweep_noalloc(n_instances, n_per_instance, B, policies, deltas, kv_cap, arrival, prompt,

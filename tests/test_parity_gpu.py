@@ -319,7 +319,7 @@ def test_invalid_arguments_rejected(S):
         S.isjl_sim_create(0, 4, 2)
 
 
-def test_sweep_equals_single_runs_and_host_entry_point(S):
+def test_sweep_equals_single_runs_and_host_entry_point(S, O):
     import torch
     from paper_2608_02244_gb300 import workloads as W
     a, p, o = W.generate(3, 8)
@@ -336,5 +336,23 @@ def test_sweep_equals_single_runs_and_host_entry_point(S):
         assert st == 0
         host = hrec.numpy().view(S.RECORD_DTYPE).reshape(len(pols), 8)
         assert host.tobytes() == res["records"].tobytes()
+    finally:
+        sm.close()
+    # with per-instance counts and upper-bound slack, through host memory
+    a, p, o, cnt = W.generate(6, 16, with_counts=True)
+    e = np.random.default_rng(3).integers(0, 50, a.shape).astype(np.int32)
+    pols, ds = ["fcfs", "ljf", "isjl", "sjf"], [0, 0, 150, 0]
+    sm = S.Simulator(16, 400, 50)
+    try:
+        res = sm.sweep(a, p, o, pols, ds, INF, counts=cnt, slack=e)
+        pin = [torch.from_numpy(np.ascontiguousarray(x)).pin_memory() for x in (a, p, o, cnt, e)]
+        hrec = torch.empty(len(pols) * 16 * S.RECORD_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
+        st = S.isjl_sim_run_sweep_host(sm.handle, pols, ds, INF, *pin[:3], hrec, h_count=pin[3], h_slack=pin[4])
+        assert st == 0
+        host = hrec.numpy().view(S.RECORD_DTYPE).reshape(len(pols), 16)
+        assert host.tobytes() == res["records"].tobytes()
+        for i, (pol, d) in enumerate(zip(pols, ds)):
+            rec, _, _ = O.run(pol, 50, d, INF, a, p, o, per_request=False, counts=cnt, slack=e)
+            assert_records_equal(host[i], rec, f"host {pol}")
     finally:
         sm.close()
