@@ -16,8 +16,9 @@
 // instantiation of the step loop), straight-line: an idle slot carries a
 // progress below 0 as a signed value and at least 2^31 as an unsigned one, so
 // the step's max (signed) and min (unsigned) need no per-slot predicate.  The
-// sum of progress over all steps is added per request when it leaves
-// (a (a + 1) / 2 for progress a).  Values that change only at events (next
+// sum of progress over all steps is added per request, o (o + 1) / 2, when it
+// starts (a run stopped early takes back the unserved part).  Values that
+// change only at events (next
 // arrival, earliest completion, start range, KV reservation) are kept as
 // warp-uniform scalars, so the steps between two events run no branch and
 // no warp reduction beyond the two of the step cost.  The pending
@@ -35,6 +36,10 @@
 // Admissions happen only at events: between events the running set, the KV
 // reservation and the queue are unchanged and A_max only grows, so a step
 // that could not start a request is followed by steps that cannot either.
+// Arrivals that cannot start anything before the next completion are released
+// at that completion, and an admission that starts several requests does so
+// up to 32 (ISJL plan entries: all) at a time, with the same outcome as one
+// start at a time.
 #include <climits>
 #include <cstdint>
 
@@ -52,7 +57,7 @@ struct WarpSmem {
     int32_t *stail;   // [B] last plan entry of worker w
     int32_t *slong;   // [B] long request o_j planned on worker j (1 <= j < n_long)
     int32_t *srem;    // [B] ISJL packing budget left on worker w (Phase ONE only)
-    int32_t *spsum;   // [B] ISJL pack sum on worker w (Phase ONE only)
+    int32_t *spsum;   // [B] ISJL pack sum on worker w in Phase ONE, then the o of its next plan entry
     int32_t *sres;    // [B] KV reserved by the request running on worker w (its planning length)
     uint32_t *pend0;  // [words0] bit p: sorted position p is pending
     uint32_t *pend1;  // [words1] bit w: pend0[w] != 0
@@ -739,11 +744,14 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             for (int w = lane; w < B; w += 32) maxrem = max(maxrem, S.srem[w]);
             maxrem = __reduce_max_sync(kFull, maxrem);
             int q = -1;
+            int64_t x_prev = -1;
+            int pos_x = 0;                                      // first sorted position with o <= x_prev
             for (;;) {
                 const int64_t x = min(theta, (int64_t)maxrem);
                 if (x < 1) break;
                 // candidates with o > x fit nowhere now or later (budgets only shrink)
-                q = bs_next(S, words0, words1, max(first_pos_le(osrt, n, x, lane), q + 1), lane);
+                if (x != x_prev) { pos_x = first_pos_le(osrt, n, x, lane); x_prev = x; }
+                q = bs_next(S, words0, words1, max(pos_x, q + 1), lane);
                 if (q >= n) break;
                 const int e = perm[q];
                 const int oe = osrt[q];
@@ -758,19 +766,24 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 int w = lowest_worker(mA, lane);                // workers M+1..B first
                 if (w < 0) w = highest_worker(mB, lane);        // then M, M-1, ..., 2
                 if (w < 0) { broken = true; return; }
+                const int remw = S.srem[w];                     // the chosen worker's budget before
+                __syncwarp();
                 if (lane == 0) {
                     const int tl = S.stail[w];
                     if (tl < 0) S.shead[w] = e; else pnext[tl] = e;
                     S.stail[w] = e;
                     pnext[e] = kNone;
+                    S.srem[w] = remw - oe;
+                    S.spsum[w] += oe;
                 }
-                if (lane == 0) { S.srem[w] -= oe; S.spsum[w] += oe; }
                 bs_clear(S, q, lane);   // includes __syncwarp
                 pend--;
                 plan_left++;
-                maxrem = -1;
-                for (int w2 = lane; w2 < B; w2 += 32) maxrem = max(maxrem, S.srem[w2]);
-                maxrem = __reduce_max_sync(kFull, maxrem);
+                if (remw == maxrem) {                            // the largest budget may have shrunk
+                    maxrem = -1;
+                    for (int w2 = lane; w2 < B; w2 += 32) maxrem = max(maxrem, S.srem[w2]);
+                    maxrem = __reduce_max_sync(kFull, maxrem);
+                }
             }
             // worker j (2..M) runs o_j after its pack
             for (int w = 1 + lane; w < nl; w += 32) {
