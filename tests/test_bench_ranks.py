@@ -48,3 +48,31 @@ def test_rank_replicas_are_independent_instances():
     assert not np.array_equal(p0, p1) and a0.shape == a1.shape
     a0b, _, _ = W.generate(3, 2)
     np.testing.assert_array_equal(a0, a0b)
+
+
+def test_reference_arm_prints_one_json_line():
+    """bench.py --impl reference times the oracle on the host and prints one
+    JSON line with the contract's keys (a small workload, one host process)."""
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--workload", "2",
+                          "--oracle-cores", "1", "--steps", "1", "--warmup", "0"],
+                         capture_output=True, text=True, timeout=300, check=True).stdout
+    lines = [l for l in out.splitlines() if l.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
+                "scaling", "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
+        assert key in d, key
+    assert d["impl"] == "reference" and d["value"] > 0 and d["cpu_baseline"]["kind"] == "oracle"
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
+
+
+def test_run_grids_are_valid():
+    import bench
+    from paper_2608_02244_gb300 import workloads as W
+    for wid, (pols, deltas, per_core) in bench.GRIDS.items():
+        assert wid in W.WORKLOADS and len(pols) == len(deltas) <= 32 and per_core >= 1
+        assert set(pols) <= {"fcfs", "ljf", "isjl", "sjf", "isjl_beta"}
