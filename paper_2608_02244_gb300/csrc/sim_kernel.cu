@@ -84,8 +84,9 @@ template <int N> struct RowCount { static constexpr int value = N; };
 
 // Row counts the step loop is instantiated for, per SPL (ascending).  The
 // loop advances the smallest of them covering every running worker; a few
-// classes keep the kernel small (measured: powers of two for SPL = 8, even
-// counts for SPL = 16), and its steps are unrolled by four.
+// classes keep the kernel small (measured: 2 and 4 for SPL = 4, 2, 4 and 8 for
+// SPL = 8, even counts for SPL = 16), and its steps are unrolled by two (four
+// for SPL = 16).
 template <int SPL> struct RowClasses;
 template <> struct RowClasses<1> {
     static constexpr int n = 1;
@@ -96,12 +97,12 @@ template <> struct RowClasses<2> {
     __host__ __device__ static constexpr int at(int i) { constexpr int v[2] = {1, 2}; return v[i]; }
 };
 template <> struct RowClasses<4> {
-    static constexpr int n = 4;
-    __host__ __device__ static constexpr int at(int i) { constexpr int v[4] = {1, 2, 3, 4}; return v[i]; }
+    static constexpr int n = 2;
+    __host__ __device__ static constexpr int at(int i) { constexpr int v[2] = {2, 4}; return v[i]; }
 };
 template <> struct RowClasses<8> {
-    static constexpr int n = 4;
-    __host__ __device__ static constexpr int at(int i) { constexpr int v[4] = {1, 2, 4, 8}; return v[i]; }
+    static constexpr int n = 3;
+    __host__ __device__ static constexpr int at(int i) { constexpr int v[3] = {2, 4, 8}; return v[i]; }
 };
 template <> struct RowClasses<16> {
     static constexpr int n = 8;
@@ -946,7 +947,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             constexpr int NR = decltype(nr_tag)::value;
             const uint32_t cnt = (uint32_t)run_cnt;
             int last_mx = 0;
-#pragma unroll 4
+            constexpr int kUnroll = SPL >= 16 ? 4 : 2;   // measured; more code costs instruction-cache misses
+#pragma unroll kUnroll
             for (int j = 0; j < L; ++j) {
                 int mx = INT_MIN;
                 unsigned mn = 0xffffffffu;
