@@ -84,9 +84,9 @@ template <int N> struct RowCount { static constexpr int value = N; };
 
 // Row counts the step loop is instantiated for, per SPL (ascending).  The
 // loop advances the smallest of them covering every running worker; a few
-// classes keep the kernel small (measured: 2 and 4 for SPL = 4, 2, 4 and 8 for
-// SPL = 8, even counts for SPL = 16), and its steps are unrolled by two (four
-// for SPL = 16).
+// classes keep the kernel small (measured: 2 and 4 for SPL = 4; 2, 4 and 8
+// for SPL = 8; 4, 8 and 16 for SPL = 16), and its steps are unrolled by two
+// (four for SPL = 16).
 template <int SPL> struct RowClasses;
 template <> struct RowClasses<1> {
     static constexpr int n = 1;
@@ -105,8 +105,8 @@ template <> struct RowClasses<8> {
     __host__ __device__ static constexpr int at(int i) { constexpr int v[3] = {2, 4, 8}; return v[i]; }
 };
 template <> struct RowClasses<16> {
-    static constexpr int n = 8;
-    __host__ __device__ static constexpr int at(int i) { constexpr int v[8] = {2, 4, 6, 8, 10, 12, 14, 16}; return v[i]; }
+    static constexpr int n = 3;
+    __host__ __device__ static constexpr int at(int i) { constexpr int v[3] = {4, 8, 16}; return v[i]; }
 };
 
 // rows advanced when the highest row holding a running worker is t - 1 (t = 0: none)
