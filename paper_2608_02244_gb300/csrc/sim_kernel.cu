@@ -535,16 +535,17 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             pend--;
             hp = bs_next(S, words0, words1, p + 1, lane);   // nothing pending below p
         };
-        // sorted positions of the first m (1 <= m <= min(32, pend)) pending
-        // requests: lane l < m gets the l-th, the other lanes -1 (uniform call)
-        auto first_pending = [&](int m) -> int {
+        // sorted positions of the first m (1 <= m <= 32) pending requests at or
+        // after position p0: lane l gets the l-th, lanes past the last one -1
+        // (uniform call)
+        auto first_pending_from = [&](int p0, int m) -> int {
             int mine = -1;
-            if (!hvalid) { hp = bs_next(S, words0, words1, 0, lane); hvalid = true; }
-            const int p0 = hp;
             for (int wb = (p0 >> 10) << 5, got = 0; got < m && wb < words0; wb += 32) {
                 if (S.pend1[wb >> 5] == 0u) continue;           // no pending in these 32 words
                 const int wi = wb + lane;
-                const uint32_t x = wi < words0 ? S.pend0[wi] : 0u;
+                uint32_t x = wi < words0 ? S.pend0[wi] : 0u;
+                if (wi < (p0 >> 5)) x = 0u;                     // below p0
+                else if (wi == (p0 >> 5)) x &= ~0u << (p0 & 31);
                 const int c = __popc(x);
                 int incl = c;
 #pragma unroll
@@ -565,6 +566,11 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 got += tot;
             }
             return mine;
+        };
+        // the first m (1 <= m <= min(32, pend)) pending requests: the longest first
+        auto first_pending = [&](int m) -> int {
+            if (!hvalid) { hp = bs_next(S, words0, words1, 0, lane); hvalid = true; }
+            return first_pending_from(hp, m);
         };
         // remove the lanes' positions p (where take) from the pending set
         auto clear_pending = [&](int p, bool take) {
@@ -857,20 +863,37 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     if (c < m) { blocked = true; break; }        // the KV cap or B stopped it
                 }
             } else if (policy == ISJL_POLICY_SJF) {
-                // shortest released request first (ties: lower index), continuous batching
-                while (run_cnt < B && pend > 0) {
+                // shortest released request first (ties: lower index), continuous
+                // batching.  The pending requests of the smallest length omin are
+                // the pending positions from the first with o <= omin upwards, in
+                // start order; one at a time for the first two starts, then up to
+                // 32 of them at a time
+                for (int nseq = 0; run_cnt < B && pend > 0;) {
                     const int hi = bs_last(S, words1, lane);
                     if (hi < 0 || hi >= n) { broken = true; return; }
                     const int omin = osrt[hi];
-                    const int p = bs_next(S, words0, words1, first_pos_le(osrt, n, omin, lane), lane);
-                    if (p >= n) { broken = true; return; }
                     if (kv_sum + omin > kv_cap) break;
-                    const int w = lowest_worker(vmask & ~busy, lane);
-                    if (w < 0) { broken = true; return; }
-                    const int e = perm[p];
-                    bs_clear(S, p, lane);
-                    pend--;
-                    start(e, omin, w);
+                    const int g = first_pos_le(osrt, n, omin, lane);
+                    if (nseq < 2) {
+                        const int p = bs_next(S, words0, words1, g, lane);
+                        if (p >= n) { broken = true; return; }
+                        const int w = lowest_worker(vmask & ~busy, lane);
+                        if (w < 0) { broken = true; return; }
+                        const int e = perm[p];
+                        bs_clear(S, p, lane);
+                        pend--;
+                        start(e, omin, w);
+                        nseq++;
+                        continue;
+                    }
+                    const int q = first_pending_from(g, min(32, pend));
+                    const int mg = __popc(__ballot_sync(kFull, q >= 0));   // of this length, in order
+                    if (mg == 0) { broken = true; return; }
+                    const int c = bulk_start(mg, q >= 0 ? perm[q] : 0, omin, vmask & ~busy);
+                    clear_pending(q, lane < c);
+                    pend -= c;
+                    hvalid = false;
+                    if (c < mg) break;
                 }
                 blocked = run_cnt >= B;
             } else if (policy == ISJL_POLICY_LJF) {
