@@ -468,7 +468,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (co_out) co_out[S.sjob[w]] = c;
             }
             busy &= ~fm;
-            if (fm) recompute_lane();
+            // unconditional where measured cheaper than the branch (not the epoch kernel's 16 rows)
+            if (!EPOCH || SPL <= 8 || fm) recompute_lane();
             if (!EPOCH) adv_rows = row_class<SPL>((int)__reduce_max_sync(kFull, 32u - (unsigned)__clz((int)busy)));
             nf = (int)__reduce_add_sync(kFull, (unsigned)nf);
             of = (int)__reduce_add_sync(kFull, (unsigned)of);
