@@ -61,9 +61,9 @@ ALU_LANES_PER_SM = 128
 OPS_PER_TOKEN_ADVANCE = 5
 OPS_PER_BATCH_STEP = 6
 # DRAM bytes (read + write) per launch of the step simulation kernel on the full
-# workload: 758.8 MB measured by ncu on the first 4,096 instances, scaled by
+# workload: 745.0 MB measured by ncu on the first 4,096 instances, scaled by
 # 10,000 / 4,096 (profiles/sim_kernel_step_online_delta_sweep_4096.md)
-SIM_DRAM_BYTES_PER_LAUNCH = 758.8e6 * 10_000 / 4_096
+SIM_DRAM_BYTES_PER_LAUNCH = 745.0e6 * 10_000 / 4_096
 
 
 def workload_config(kernel, wl, n_inst, policies, deltas, flush):
