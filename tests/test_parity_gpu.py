@@ -302,6 +302,26 @@ def test_step_limit_partial_records(S, O, epoch):
         assert (res["start"] == -1).any() and (res["completion"] == -1).any()
 
 
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_bulk_starts_with_ties_and_partial_rows(S, O, epoch):
+    """Admissions that start many requests at once (the 32-wide bulk path):
+    lengths from a tiny set (long runs of equal o, so SJF and LJF take large
+    tie groups in index order), B spanning several register rows with a
+    partial last row, every request at t = 0 or in bursts, with and without a
+    KV cap that stops a bulk in its middle."""
+    rng = np.random.default_rng(21)
+    n = 300
+    a = np.zeros((6, n), np.int32)
+    a[3:] = np.sort(rng.integers(0, 40, (3, n)), axis=1)          # bursts of arrivals
+    p = np.zeros((6, n), np.int32)
+    o = rng.choice(np.array([3, 7, 7, 12, 40], np.int32), (6, n)).astype(np.int32)
+    pols = ["fcfs", "ljf", "sjf", "isjl", "isjl", "isjl", "isjl_beta"]
+    ds = [0, 0, 0, 4, 30, INF, 8]
+    for B in (33, 100, 256):
+        for kv in (INF, 700):
+            run_both(S, O, a, p, o, B, pols, ds, kv, epoch)
+
+
 def test_invalid_arguments_rejected(S):
     import torch
     sm = S.Simulator(1, 4, 2)
