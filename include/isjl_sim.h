@@ -50,7 +50,10 @@ typedef enum {
     ISJL_ERR_OOM = 3,          /* device or pinned-host allocation failed in create / first host call */
     ISJL_ERR_CUDA = 4,         /* a CUDA runtime call failed (launch, copy, sync) */
     ISJL_ERR_STEP_LIMIT = 5,   /* a simulation exceeded max_steps (defensive guard; never trapped) */
-    ISJL_ERR_NOT_READY = 6     /* metrics requested before any run */
+    ISJL_ERR_NOT_READY = 6,    /* metrics requested before any run */
+    ISJL_ERR_INTERNAL = 7      /* an internal invariant of the simulation kernel failed (a library bug):
+                                  the run stopped where it found it; its counters are partial and its
+                                  per-request outputs -1 beyond what it had written */
 } isjl_status;
 
 typedef enum {

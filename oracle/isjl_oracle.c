@@ -78,6 +78,8 @@ typedef struct {
     int64_t t0, d1;
     int32_t L1;               /* o_1 of the current stage (worker 1) */
     int32_t *long_of;         /* long_of[j]: o_j planned on worker j, 2..M */
+    int flags;                /* ISJL reading variants (0 = the specified readings) */
+    int broke;                /* the gate kept a free worker from a queued request */
 } sim_t;
 
 /* ---- sorting by (o desc, idx asc) --------------------------------------- */
@@ -188,6 +190,30 @@ static void ljf_admit(sim_t *s, int64_t k) {
 }
 
 /* ---- ISJL (Algorithm 2 with beta = alpha; online rolling form, Sec. 3.4) - */
+/*
+ * State: every worker is running a request, holds plan entries (reserved) or
+ * is free.  A stage starts when nothing runs, no plan entry is left and the
+ * released queue Q(k) is nonempty.  Phase ONE then fixes a plan: worker 1
+ * gets the longest request o_1, to be started d1 steps after the stage start;
+ * worker j in 2..M gets a pack of shorter requests followed by the j-th
+ * longest request o_j; workers beyond M get a pack only.  Every start, planned
+ * or not, needs the fairness gate A_max(k) <= alpha (Eq. 1: a request starts
+ * at progress 0, so the gap it opens is the largest running progress) and the
+ * KV reservation.  Phase TWO gives free workers the longest released request.
+ *
+ * The reading variants below exist only for the reading study (each is off by
+ * default and none is part of the specified path):
+ */
+#define V_NO_WAIT_O1     1    /* o_j may start before o_1 has started */
+#define V_D1_LAST        2    /* d1 from the pack of worker M alone */
+#define V_P2_RESERVED    4    /* Phase TWO may use a worker whose plan entry waits */
+#define V_REBUILD_REOPEN 8    /* new Phase ONE once the gate reopens after stopping Phase TWO */
+#define V_LITERAL_LONG  16    /* o_2..o_M are not planned: packs scan every shorter request, Phase TWO starts the rest */
+#define V_SHORT_PACKS   32    /* packs take only requests with o <= alpha */
+#define V_CANCEL        64    /* a plan stopped by the gate goes back to the queue */
+#define V_WAIVER       128    /* o_1's delay is skipped at a later step that finds nothing running */
+#define V_UNGATED_PLAN 256    /* plan entries start without the gate (breaks Eq. 1; for contrast) */
+
 static void plan_append(sim_t *s, int j, int32_t i) {
     s->status[i] = ST_PLANNED;
     s->plan_next[i] = -1;
@@ -196,108 +222,149 @@ static void plan_append(sim_t *s, int j, int32_t i) {
     s->plan_left++;
 }
 
-/* Phase ONE at a stage start (nothing runs, no plan entry is left, and the
- * released queue Q(k) is nonempty).  Returns 1 if a plan was made. */
-static int isjl_phase_one(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_t *budget) {
+/* Phase ONE over the workers wk[0..nw-1] (wk[0] plays worker 1, wk[j-1]
+ * worker j).  Returns 1 if a plan was made, 0 if the stage goes straight to
+ * Phase TWO (|Q| = 1, or the second longest request is no longer than alpha). */
+static int isjl_phase_one(sim_t *s, int64_t k, const int32_t *wk, int nw, int32_t *Q, int64_t *packsum,
+                          int64_t *budget, int32_t *visit) {
     const int64_t al = s->alpha;
+    const int64_t be = s->beta;   /* beta = alpha (Algorithm 2), or Algorithm "ISJL"'s beta */
     int q = 0;
-    /* Q(k) in the order o_1 >= o_2 >= ... (ties: lower index first) */
-    for (int p = 0; p < s->n; ++p) {
+    for (int p = 0; p < s->n; ++p) {            /* Q(k) longest first, ties by index */
         int32_t i = s->by_len[p];
         if (s->status[i] == ST_WAIT && s->arr[i] <= k) Q[q++] = i;
     }
     s->t0 = k;
     s->d1 = 0;
     s->L1 = -1;
-    /* |Q| = 1 or o_2 <= alpha: go straight to Phase TWO */
     if (q < 2 || (int64_t)s->o[Q[1]] <= al) return 0;
 
-    /* M = min{B, #{o_i > alpha}}  (called n_long to avoid the KV-cap clash) */
-    int cnt_long = 0;
-    for (int p = 0; p < q; ++p) if ((int64_t)s->o[Q[p]] > al) cnt_long++;
-    int n_long = cnt_long < s->B ? cnt_long : s->B;
+    /* M: how many of the B workers take a long request (o > alpha) */
+    int n_long = 0;
+    for (int p = 0; p < q && n_long < nw; ++p) if ((int64_t)s->o[Q[p]] > al) n_long++;
     const int64_t o1 = s->o[Q[0]];
-    const int64_t be = s->beta;   /* beta = alpha (Algorithm 2), or Algorithm "ISJL"'s beta */
-    const int64_t theta = min64(2 * al, o1 - (int64_t)s->o[Q[n_long - 1]] + be);
+    /* a pack member is at most theta = min{2 alpha, o_1 - o_M + beta} long
+     * (for the short-packs variant also at most alpha) */
+    int64_t theta = min64(2 * al, o1 - (int64_t)s->o[Q[n_long - 1]] + be);
+    if (s->flags & V_SHORT_PACKS) theta = min64(theta, al);
 
-    /* packing budgets: workers 2..M get cap_j = min{2 alpha, o_1 - o_j + beta},
-     * workers M+1..B get alpha */
-    for (int j = 1; j <= s->B; ++j) { packsum[j] = 0; budget[j] = -1; }
-    for (int j = 2; j <= n_long; ++j) budget[j] = min64(2 * al, o1 - (int64_t)s->o[Q[j - 1]] + be);
-    for (int j = n_long + 1; j <= s->B; ++j) budget[j] = al;
+    /* pack budgets: alpha on a worker without a long request; on worker j
+     * (2 <= j <= M) the room that lets o_j still end within beta of o_1,
+     * capped at 2 alpha.  Visiting order of the first fit: the workers without
+     * a long request first, then the long ones from o_M back to o_2. */
+    int nv = 0;
+    for (int j = 1; j <= nw; ++j) { packsum[j] = 0; budget[j] = -1; }
+    for (int j = n_long + 1; j <= nw; ++j) { budget[j] = al; visit[nv++] = j; }
+    for (int j = n_long; j >= 2; --j) {
+        budget[j] = min64(2 * al, o1 - (int64_t)s->o[Q[j - 1]] + be);
+        visit[nv++] = j;
+    }
+    const int literal = (s->flags & V_LITERAL_LONG) != 0;
+    s->status[Q[0]] = ST_PLANNED;
+    if (!literal) for (int p = 1; p < n_long; ++p) s->status[Q[p]] = ST_PLANNED;
 
-    /* the long requests leave the queue (worker j will run o_j) */
-    for (int p = 0; p < n_long; ++p) s->status[Q[p]] = ST_PLANNED;
-
-    /* first fit of the short requests o_i <= theta that follow the long ones,
-     * in sorted order: workers M+1..B (budget alpha) first, then workers
-     * M, M-1, ..., 2 (budget cap_j).  A request that fits nowhere stays in Q. */
-    for (int p = n_long; p < q; ++p) {
+    /* first fit, longest candidate first; a candidate that fits nowhere stays queued */
+    for (int p = literal ? 1 : n_long; p < q; ++p) {
         int32_t i = Q[p];
         int64_t oi = s->o[i];
         if (oi > theta) continue;
-        int placed = 0;
-        for (int j = n_long + 1; j <= s->B && !placed; ++j)
-            if (oi + packsum[j] <= budget[j]) { plan_append(s, j, i); packsum[j] += oi; placed = 1; }
-        for (int j = n_long; j >= 2 && !placed; --j)
-            if (oi + packsum[j] <= budget[j]) { plan_append(s, j, i); packsum[j] += oi; placed = 1; }
+        for (int v = 0; v < nv; ++v) {
+            int j = visit[v];
+            if (packsum[j] + oi <= budget[j]) { plan_append(s, wk[j - 1], i); packsum[j] += oi; break; }
+        }
     }
-    /* worker 1 runs o_1; worker j in 2..M runs its pack, then o_j */
-    plan_append(s, 1, Q[0]);
+    /* worker 1 holds o_1; worker j (2..M) runs o_j after its pack */
+    plan_append(s, wk[0], Q[0]);
     s->L1 = Q[0];
     for (int j = 0; j <= s->B; ++j) s->long_of[j] = -1;
-    for (int j = 2; j <= n_long; ++j) { plan_append(s, j, Q[j - 1]); s->long_of[j] = Q[j - 1]; }
+    if (!literal)
+        for (int j = 2; j <= n_long; ++j) { plan_append(s, wk[j - 1], Q[j - 1]); s->long_of[wk[j - 1]] = Q[j - 1]; }
 
-    /* o_1 waits d1 = min{max{max_j sum(w_j) - alpha, 0}, alpha} steps, j = 2..M */
+    /* d1: the smallest delay after which o_1's progress is at most alpha when
+     * the longest pack ends, min{max{max_j sum(w_j) - alpha, 0}, alpha} over
+     * j = 2..M (the last-pack variant uses worker M's pack alone) */
     int64_t mx = 0;
-    for (int j = 2; j <= n_long; ++j) mx = max64(mx, packsum[j]);
+    if (s->flags & V_D1_LAST) mx = n_long >= 2 ? packsum[n_long] : 0;
+    else for (int j = 2; j <= n_long; ++j) mx = max64(mx, packsum[j]);
     s->d1 = min64(max64(mx - al, 0), al);
     return 1;
 }
 
+static int worker_free(const sim_t *s, int j) { return s->worker_job[j] < 0 && s->plan_head[j] < 0; }
+
 /* ISJL admission for step k:
- *   1. stage start (Phase ONE) when nothing runs, no plan entry is left and
- *      Q(k) is nonempty;
- *   2. plan starts, workers 1..B in order: an idle worker with plan entries
- *      starts its next entry if A_max(k) <= alpha and the KV reservation fits;
- *      worker 1's o_1 also waits until k >= t0 + d1 (waived once a later step
- *      finds nothing running), and a long request o_j (j >= 2) also waits
- *      until o_1 has started (Section 3.3: the pack tails run "in parallel
- *      with o_1", and o_j follows its pack).  A blocked entry waits on its
- *      worker;
- *   3. Phase TWO: while a worker is free (not running, no plan entries), Q(k)
- *      is nonempty and A_max(k) <= alpha, start the longest released request.
- * Requests arriving during a stage only join Q(k) (never the current plan).
- * A start always has progress 0, so A_max(k) is the same for every start of
- * the step. */
-static void isjl_admit(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_t *budget) {
+ *   1. a stage start runs Phase ONE;
+ *   2. plan starts, workers 1..B in order: a worker that is not running starts
+ *      its next plan entry if the gate and the KV reservation allow it; o_1
+ *      also waits until k >= t0 + d1, and o_j (j >= 2) until o_1 has started
+ *      (the pack runs alone, o_1 joins it, o_j follows the pack alongside
+ *      o_1 -- Section 3.2's order, kept by Section 3.3's stages, which hold
+ *      o_1 on worker 1 while the packs run).  An entry that cannot start
+ *      waits on its worker;
+ *   3. Phase TWO: while a worker is free, Q(k) is nonempty and the gate is
+ *      open, the longest released request starts on the lowest free worker.
+ * The first KV failure ends the step's starts.  Requests arriving during a
+ * stage only join Q(k).  Starts have progress 0, so A_max(k) is the same for
+ * every start of the step. */
+static void isjl_admit(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_t *budget, int32_t *wk) {
     const int nothing_runs = (s->run_cnt == 0);
-    if (nothing_runs && s->plan_left == 0 && longest_waiting(s, k) >= 0)
-        isjl_phase_one(s, k, Q, packsum, budget);
+    const int64_t amax = a_max(s);
+    if (s->plan_left == 0 && longest_waiting(s, k) >= 0) {
+        int nw = 0;
+        if (nothing_runs) {
+            for (int j = 1; j <= s->B; ++j) wk[nw++] = j;
+        } else if ((s->flags & V_REBUILD_REOPEN) && s->broke && amax <= s->alpha) {
+            for (int j = 1; j <= s->B; ++j) if (worker_free(s, j)) wk[nw++] = j;
+        }
+        if (nw > 0) {
+            isjl_phase_one(s, k, wk, nw, Q, packsum, budget, wk + s->B + 1);
+            s->broke = 0;
+        }
+    }
 
-    const int gate_ok = a_max(s) <= s->alpha;
-    int stop = !gate_ok;
-
+    const int gate_ok = amax <= s->alpha;
+    int stop = 0;
     for (int j = 1; j <= s->B && !stop; ++j) {
         int32_t e = s->plan_head[j];
         if (e < 0 || s->worker_job[j] >= 0) continue;
-        if (j == 1 && e == s->L1) {
-            int delay_over = (k >= s->t0 + s->d1) || (k > s->t0 && nothing_runs);
-            if (!delay_over) continue;
+        if (!gate_ok && !(s->flags & V_UNGATED_PLAN)) {
+            stop = 1;
+            if (s->flags & V_CANCEL) {             /* the plan goes back to the queue */
+                for (int w = 1; w <= s->B; ++w) {
+                    for (int32_t x = s->plan_head[w]; x >= 0; x = s->plan_next[x]) s->status[x] = ST_WAIT;
+                    s->plan_head[w] = s->plan_tail[w] = -1;
+                    s->long_of[w] = -1;
+                }
+                s->plan_left = 0;
+                s->L1 = -1;
+            }
+            break;
         }
-        if (j >= 2 && e == s->long_of[j] && s->status[s->L1] == ST_PLANNED) continue;
+        if (e == s->L1) {
+            int over = k >= s->t0 + s->d1;
+            if ((s->flags & V_WAIVER) && k > s->t0 && nothing_runs) over = 1;
+            if (!over) continue;
+        }
+        if (e == s->long_of[j] && s->L1 >= 0 && s->status[s->L1] == ST_PLANNED && !(s->flags & V_NO_WAIT_O1))
+            continue;
         if (s->kv_sum + s->o[e] > s->kv_cap) { stop = 1; break; }
         s->plan_head[j] = s->plan_next[e];
         if (s->plan_head[j] < 0) s->plan_tail[j] = -1;
         s->plan_left--;
         start_job(s, e, k, j);
     }
-    if (stop) return;
+    if (stop || !gate_ok) {
+        /* a free worker and a queued request that the closed gate keeps apart */
+        if (!gate_ok && longest_waiting(s, k) >= 0)
+            for (int j = 1; j <= s->B; ++j) if (worker_free(s, j)) { s->broke = 1; break; }
+        return;
+    }
 
     for (;;) {
         int w = -1;
-        for (int j = 1; j <= s->B; ++j)
-            if (s->worker_job[j] < 0 && s->plan_head[j] < 0) { w = j; break; }
+        for (int j = 1; j <= s->B && w < 0; ++j) if (worker_free(s, j)) w = j;
+        if (w < 0 && (s->flags & V_P2_RESERVED))
+            for (int j = 1; j <= s->B && w < 0; ++j) if (s->worker_job[j] < 0) w = j;
         if (w < 0) break;
         int32_t i = longest_waiting(s, k);
         if (i < 0) break;
@@ -310,10 +377,10 @@ static void isjl_admit(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_
 /* Simulate one instance under one policy.  delta is the fairness budget
  * (INT32_MAX = no constraint; ignored by FCFS and LJF except for counting
  * violations).  start_out/compl_out may be NULL.  Returns the status. */
-int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
-               const int32_t *arrival, const int32_t *prompt, const int32_t *output, const int32_t *slack,
-               double c, double tau, double p0, int64_t max_steps,
-               int32_t *start_out, int32_t *compl_out, or_record *rec)
+int oracle_run_v(int policy, int B, int64_t delta, int64_t kv_cap, int n,
+                 const int32_t *arrival, const int32_t *prompt, const int32_t *output, const int32_t *slack,
+                 double c, double tau, double p0, int64_t max_steps, int flags,
+                 int32_t *start_out, int32_t *compl_out, or_record *rec)
 {
     memset(rec, 0, sizeof(*rec));
     if (n < 0 || B < 1 || delta < 0 || kv_cap < 1 || policy < 0 || policy > 4 || (n > 0 && (!arrival || !prompt || !output))) {
@@ -330,7 +397,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     sim_t *s = &S;
     s->n = n; s->B = B; s->policy = policy == OR_ISJL_BETA ? OR_ISJL : policy; s->alpha = delta;
     s->beta = policy == OR_ISJL_BETA ? beta_of(delta) : delta;
-    s->kv_cap = kv_cap; s->arr = arrival;
+    s->kv_cap = kv_cap; s->arr = arrival; s->flags = flags;
     policy = s->policy;
     s->o = malloc(sizeof(int32_t) * n);
     s->ot = malloc(sizeof(int32_t) * n);
@@ -343,6 +410,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     int32_t *Q = malloc(sizeof(int32_t) * n);
     int64_t *packsum = malloc(sizeof(int64_t) * (size_t)(B + 1));
     int64_t *budget = malloc(sizeof(int64_t) * (size_t)(B + 1));
+    int32_t *wk = malloc(sizeof(int32_t) * (size_t)(2 * B + 2));   /* stage workers, then the first-fit order */
     s->worker_job = malloc(sizeof(int32_t) * (size_t)(B + 1));
     s->plan_head = malloc(sizeof(int32_t) * (size_t)(B + 1));
     s->plan_tail = malloc(sizeof(int32_t) * (size_t)(B + 1));
@@ -351,7 +419,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
     s->long_of = malloc(sizeof(int32_t) * (size_t)(B + 1));
     int status = OR_OK;
     if (!s->o || !s->ot || !s->status || !s->a || !s->start || !s->compl || !s->by_len || !s->run || !Q ||
-        !packsum || !budget || !s->worker_job || !s->plan_head || !s->plan_tail || !s->plan_next || !s->job_worker || !s->long_of) {
+        !packsum || !budget || !wk || !s->worker_job || !s->plan_head || !s->plan_tail || !s->plan_next || !s->job_worker || !s->long_of) {
         status = OR_OOM; goto done;
     }
 
@@ -405,7 +473,7 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
         if (policy == OR_FCFS) fcfs_admit(s, k);
         else if (policy == OR_LJF) ljf_admit(s, k);
         else if (policy == OR_SJF) sjf_admit(s, k);
-        else isjl_admit(s, k, Q, packsum, budget);
+        else isjl_admit(s, k, Q, packsum, budget, wk);
 
         /* serve step k: every running request processes token r_i = a_i + 1 */
         if (s->run_cnt > 0) {
@@ -452,28 +520,49 @@ int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
 done:
     rec->status = status;
     free(s->o); free(s->ot); free(s->status); free(s->a); free(s->start); free(s->compl); free(s->by_len);
-    free(s->run); free(Q); free(packsum); free(budget); free(s->worker_job); free(s->plan_head);
+    free(s->run); free(Q); free(packsum); free(budget); free(wk); free(s->worker_job); free(s->plan_head);
     free(s->plan_tail); free(s->plan_next); free(s->job_worker); free(s->long_of);
     return status;
 }
 
-/* Run many instances (row-major, n per row) under one (policy, delta).
+/* The run with the specified readings (no variant flags). */
+int oracle_run(int policy, int B, int64_t delta, int64_t kv_cap, int n,
+               const int32_t *arrival, const int32_t *prompt, const int32_t *output, const int32_t *slack,
+               double c, double tau, double p0, int64_t max_steps,
+               int32_t *start_out, int32_t *compl_out, or_record *rec)
+{
+    return oracle_run_v(policy, B, delta, kv_cap, n, arrival, prompt, output, slack, c, tau, p0, max_steps, 0,
+                        start_out, compl_out, rec);
+}
+
+/* Run many instances (row-major, n per row) under one (policy, delta) and
+ * the ISJL reading variants `flags` (0: the specified readings).
  * rec has n_inst entries; start_out/compl_out are n_inst*n or NULL.
  * Returns the first nonzero status, else 0. */
+int oracle_run_batch_v(int policy, int B, int64_t delta, int64_t kv_cap, int n_inst, int n,
+                       const int32_t *arrival, const int32_t *prompt, const int32_t *output, const int32_t *slack,
+                       double c, double tau, double p0, int64_t max_steps, int flags,
+                       int32_t *start_out, int32_t *compl_out, or_record *rec)
+{
+    int first = 0;
+    for (int t = 0; t < n_inst; ++t) {
+        size_t off = (size_t)t * (size_t)n;
+        int st = oracle_run_v(policy, B, delta, kv_cap, n, arrival + off, prompt + off, output + off,
+                              slack ? slack + off : NULL, c, tau, p0, max_steps, flags,
+                              start_out ? start_out + off : NULL, compl_out ? compl_out + off : NULL, rec + t);
+        if (st && !first) first = st;
+    }
+    return first;
+}
+
+/* Run many instances under one (policy, delta) with the specified readings. */
 int oracle_run_batch(int policy, int B, int64_t delta, int64_t kv_cap, int n_inst, int n,
                      const int32_t *arrival, const int32_t *prompt, const int32_t *output, const int32_t *slack,
                      double c, double tau, double p0, int64_t max_steps,
                      int32_t *start_out, int32_t *compl_out, or_record *rec)
 {
-    int first = 0;
-    for (int t = 0; t < n_inst; ++t) {
-        size_t off = (size_t)t * (size_t)n;
-        int st = oracle_run(policy, B, delta, kv_cap, n, arrival + off, prompt + off, output + off,
-                            slack ? slack + off : NULL, c, tau, p0, max_steps, start_out ? start_out + off : NULL,
-                            compl_out ? compl_out + off : NULL, rec + t);
-        if (st && !first) first = st;
-    }
-    return first;
+    return oracle_run_batch_v(policy, B, delta, kv_cap, n_inst, n, arrival, prompt, output, slack, c, tau, p0,
+                              max_steps, 0, start_out, compl_out, rec);
 }
 
 int oracle_record_size(void) { return (int)sizeof(or_record); }

@@ -44,6 +44,11 @@ def lib():
                                        ctypes.c_double, ctypes.c_double, ctypes.c_double,
                                        ctypes.c_int64, p32, p32, ctypes.c_void_p]
         L.oracle_run_batch.restype = ctypes.c_int
+        L.oracle_run_batch_v.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
+                                         ctypes.c_int, ctypes.c_int, p32, p32, p32, p32,
+                                         ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                         ctypes.c_int64, ctypes.c_int, p32, p32, ctypes.c_void_p]
+        L.oracle_run_batch_v.restype = ctypes.c_int
         L.oracle_record_size.restype = ctypes.c_int
         L.oracle_beta.argtypes = [ctypes.c_int64]
         L.oracle_beta.restype = ctypes.c_int64
@@ -64,8 +69,13 @@ def _ptr(a):
     return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
 
 
+# ISJL reading variants (the reading study only; 0 = the specified readings)
+VARIANTS = {"no_wait_o1": 1, "d1_last": 2, "p2_reserved": 4, "rebuild_reopen": 8, "literal_long": 16,
+            "short_packs": 32, "cancel": 64, "waiver": 128, "ungated_plan": 256}
+
+
 def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p0=0.002,
-        max_steps=0, per_request=True, counts=None, slack=None):
+        max_steps=0, per_request=True, counts=None, slack=None, variant=0):
     """Simulate every instance (row) under one policy and budget.
 
     Returns (records, start, completion); records is a structured array with
@@ -75,6 +85,8 @@ def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p
     counts[i] requests (ragged batches); the rest stay -1.  ``slack`` (optional,
     shaped like ``arrival``) is the upper-bound slack e_i = u_i - o_i: policies
     plan with u_i and requests finish after o_i tokens (Robust-ISJL).
+    ``variant`` ORs VARIANTS flags: alternative readings of Algorithm 2, used
+    only by the reading study; 0 is the simulator's specification.
     """
     if counts is not None:
         a, p, o = (np.atleast_2d(_i32(x)) for x in (arrival, prompt, output))
@@ -91,7 +103,8 @@ def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p
                     cos.append(np.full((1, a.shape[1]), -1, np.int32))
                 continue
             r, st, co = run(policy, B, delta, kv_cap, a[i:i + 1, :m], p[i:i + 1, :m], o[i:i + 1, :m], c, tau, p0,
-                            max_steps, per_request, slack=e[i:i + 1, :m] if e is not None else None)
+                            max_steps, per_request, slack=e[i:i + 1, :m] if e is not None else None,
+                            variant=variant)
             recs.append(r)
             if per_request:
                 row = np.full((1, a.shape[1]), -1, np.int32)
@@ -112,11 +125,11 @@ def run(policy, B, delta, kv_cap, arrival, prompt, output, c=0.0005, tau=1e-6, p
     rec = np.zeros(n_inst, RECORD_DTYPE)
     st = np.full((n_inst, n), -1, np.int32) if per_request else None
     co = np.full((n_inst, n), -1, np.int32) if per_request else None
-    lib().oracle_run_batch(POLICIES[policy], int(B), int(delta), int(kv_cap), n_inst, n,
-                           _ptr(a), _ptr(p), _ptr(o), _ptr(e) if e is not None else None,
-                           float(c), float(tau), float(p0), int(max_steps),
-                           _ptr(st) if per_request else None, _ptr(co) if per_request else None,
-                           rec.ctypes.data)
+    lib().oracle_run_batch_v(POLICIES[policy], int(B), int(delta), int(kv_cap), n_inst, n,
+                             _ptr(a), _ptr(p), _ptr(o), _ptr(e) if e is not None else None,
+                             float(c), float(tau), float(p0), int(max_steps), int(variant),
+                             _ptr(st) if per_request else None, _ptr(co) if per_request else None,
+                             rec.ctypes.data)
     if squeeze:
         rec = rec[0]
         st = st[0] if per_request else None

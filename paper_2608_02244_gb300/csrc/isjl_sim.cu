@@ -74,6 +74,7 @@ const char *isjl_status_string(isjl_status st) {
         case ISJL_ERR_CUDA: return "CUDA runtime error";
         case ISJL_ERR_STEP_LIMIT: return "step limit exceeded";
         case ISJL_ERR_NOT_READY: return "no run to report";
+        case ISJL_ERR_INTERNAL: return "internal invariant failed (library bug)";
     }
     return "unknown status";
 }

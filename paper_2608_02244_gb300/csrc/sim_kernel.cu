@@ -914,13 +914,13 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     uint32_t cand = resv & ~busy;
                     if (!L1_started) {
                         cand &= ~lhead;
-                        const bool over = ((int64_t)k >= (int64_t)t0 + d1) || (k > t0 && nothing_runs);
+                        const bool over = (int64_t)k >= (int64_t)t0 + d1;
                         if (!over && lane == 0) cand &= ~1u;        // worker 0 holds o_1
                     }
                     for (int nseq = 0;;) {
                         if (nseq >= 2) {                            // the rest at once
                             if (__ballot_sync(kFull, cand != 0u)) {
-                                const bool over = ((int64_t)k >= (int64_t)t0 + d1) || (k > t0 && nothing_runs);
+                                const bool over = (int64_t)k >= (int64_t)t0 + d1;
                                 stop = plan_bulk(cand, over);
                             }
                             break;
@@ -930,7 +930,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         if (lane == (w & 31)) cand &= ~(1u << (w >> 5));
                         const int e = S.shead[w];
                         if (w == 0 && e == L1) {
-                            const bool over = ((int64_t)k >= (int64_t)t0 + d1) || (k > t0 && nothing_runs);
+                            const bool over = (int64_t)k >= (int64_t)t0 + d1;
                             if (!over) continue;                 // o_1 still delayed
                         }
                         if (w >= 1 && w < nlong && e == S.slong[w] && !L1_started) continue;  // o_j after o_1
@@ -1006,7 +1006,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     if (done == n) break;
                     if (k >= next_arr) release();
                     admit();
-                    if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
+                    if (broken) { status = ISJL_ERR_INTERNAL; break; }
                     next_check = blocked && run_cnt > 0 ? INT_MAX : next_arr;
                     if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) next_check = min(next_check, t0 + d1);
                     next_check = min(next_check, step_guard);
@@ -1020,7 +1020,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     if (adv_rows < 1) broken = true;
                     else dispatch_rows<SPL, 0, RowClasses<SPL>::n - 1>(adv_rows, f);
                 }
-                if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
+                if (broken) { status = ISJL_ERR_INTERNAL; break; }
                 Tb += L;
                 tok += L * run_cnt;
                 if (kv_over) kvviol += L;
@@ -1048,7 +1048,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (k == cmin) retire(k);
                 if (done == n) break;
                 admit();
-                if (broken) { status = ISJL_ERR_STEP_LIMIT; break; }
+                if (broken) { status = ISJL_ERR_INTERNAL; break; }
                 // next event: arrival, completion or the end of o_1's delay
                 int32_t nxt = min(blocked && run_cnt > 0 ? INT_MAX : next_arr, cmin);
                 if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) nxt = min(nxt, t0 + d1);

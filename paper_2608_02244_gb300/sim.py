@@ -18,7 +18,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "_build", "libisjl_sim.so")
 
 ISJL_OK, ISJL_ERR_INVALID_ARG, ISJL_ERR_INFEASIBLE, ISJL_ERR_OOM = 0, 1, 2, 3
-ISJL_ERR_CUDA, ISJL_ERR_STEP_LIMIT, ISJL_ERR_NOT_READY = 4, 5, 6
+ISJL_ERR_CUDA, ISJL_ERR_STEP_LIMIT, ISJL_ERR_NOT_READY, ISJL_ERR_INTERNAL = 4, 5, 6, 7
 POLICY = {"fcfs": 0, "ljf": 1, "isjl": 2, "sjf": 3, "isjl_beta": 4}
 DELTA_INF = 2**31 - 1
 KV_INF = 2**31 - 1

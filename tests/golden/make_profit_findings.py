@@ -21,11 +21,25 @@ ROOT = os.path.dirname(os.path.dirname(HERE))
 sys.path.insert(0, ROOT)
 
 from oracle import oracle as O  # noqa: E402
-from paper_2608_02244_gb300 import analysis, workloads as W  # noqa: E402
+from paper_2608_02244_gb300 import workloads as W  # noqa: E402
 
 INF = 2**31 - 1
 REPS = 200
 KEYS = [("fcfs", 0), ("ljf", 0)] + [("isjl", a) for a in W.WORKLOADS[6].deltas]
+
+
+COLS = ("profit", "cost", "tau_Q", "c_T", "tau_E", "throughput", "avg_extent")
+
+
+def means(rec):
+    """Means over replications of Table 1's columns, taken from oracle records:
+    the average extent of a replication is its sum of step extents over its
+    nonempty steps."""
+    row = {c: float(np.mean(rec[c])) for c in COLS if c != "avg_extent"}
+    tb = rec["T_busy"].astype(np.float64)
+    row["avg_extent"] = float(np.mean(rec["sum_extent"] / np.maximum(tb, 1.0)))
+    row["T_make"] = float(np.mean(rec["T_make"]))
+    return row
 
 
 def compute(reps=REPS):
@@ -34,7 +48,7 @@ def compute(reps=REPS):
     for pol, d in KEYS:
         rec, _, _ = O.run(pol, 50, d, INF, a, p, o, per_request=False, counts=cnt)
         recs[(pol, d)] = rec
-    return recs, analysis.cost_table(recs, ljf_key=("ljf", 0))
+    return recs, {k: means(r) for k, r in recs.items()}
 
 
 def main():
@@ -45,7 +59,7 @@ def main():
                 "# (Section 5.2 design; B = 50, no KV cap).  Written by make_profit_findings.py.\n"
                 "# columns: policy alpha profit cost tau_Q c_T tau_E throughput avg_extent T_make\n")
         for (pol, d), row in table.items():
-            vals = [row[k] for k in analysis.TABLE1_FIELDS] + [row["T_make"]]
+            vals = [row[k] for k in COLS] + [row["T_make"]]
             f.write(f"{pol} {d} " + " ".join(f"{v:.10g}" for v in vals) + "\n")
     print(path)
 
