@@ -53,13 +53,24 @@ GRIDS = {
     6: (["fcfs", "ljf"] + ["isjl"] * 7, [0, 0, 50, 100, 150, 250, 300, 400, 500], 400),
     8: (["fcfs", "ljf", "isjl", "isjl", "isjl", "isjl", "isjl"], [0, 0, 16, 64, 256, 1024, INF], 40),
 }
-# int32 ALU lanes per SM on GB300 (4 SM sub-partitions x 32 lanes) and SM count
+# nominal int32 lanes per SM on GB300 (4 SM sub-partitions x 32 lanes), for context
 ALU_LANES_PER_SM = 128
 # algorithmic integer work of the per-step kernel: per token-advance
 # (r = a + 1, store, max, min, add/compare) and per batch-step (W, E, extent,
 # violation, T_busy, token counter)
 OPS_PER_TOKEN_ADVANCE = 5
 OPS_PER_BATCH_STEP = 6
+# algorithmic integer work of the event-driven kernel: per request start or
+# completion (KV reservation, earliest completion / start range, counter,
+# output store, queue bit) and per epoch, a step at which a request starts or
+# completes (the closed-form W, E, extent, max extent, violations, T_busy and
+# token terms of the interval that follows)
+OPS_PER_REQUEST_EVENT = 5
+OPS_PER_EPOCH = 14
+# probe launches for the measured integer rates: iterations per thread (about
+# 30-60 ms per launch on GB300) and launches per kind (the fastest is kept)
+PROBE_ITERS = 20_000
+PROBE_LAUNCHES = 3
 # DRAM bytes (read + write) per launch of the step simulation kernel on the full
 # workload: 745.0 MB measured by ncu on the first 4,096 instances, scaled by
 # 10,000 / 4,096 (profiles/sim_kernel_step_online_delta_sweep_4096.md)
@@ -119,6 +130,35 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(smax) if smax else None,
                 "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------ measured peaks ----
+def probe_peaks(sim, stream):
+    """Measured int32 issue rates (Tops/s): adds and min / max, best of
+    PROBE_LAUNCHES launches each (isjl_probe_int_rate)."""
+    out = {}
+    for kind, name in ((0, "add"), (1, "minmax")):
+        best = 0.0
+        for _ in range(PROBE_LAUNCHES):
+            n, ms = sim.isjl_probe_int_rate(kind, PROBE_ITERS, stream)
+            best = max(best, n / (ms / 1e3) / 1e12)
+        out[name] = best
+    return out
+
+
+def epoch_count(start, completion):
+    """Steps at which some request starts or completes, summed over (run,
+    instance): the epochs the event-driven kernel closes in closed form."""
+    runs = start.shape[0]
+    total = 0
+    for r in range(runs):
+        ev = np.concatenate([start[r], completion[r]], axis=1)
+        ev = np.sort(ev, axis=1)
+        valid = ev >= 0
+        new = np.ones_like(valid)
+        new[:, 1:] = ev[:, 1:] != ev[:, :-1]
+        total += int((valid & new).sum())
+    return total
 
 
 # ------------------------------------------------------------ CPU oracle ----
@@ -380,26 +420,49 @@ def main():
         return 0
 
     value = units_all / (t_ms_all / 1e3)
-    sim_avg_ms = sum(sim_ms) / len(sim_ms)
     sm_mhz = clocks.get("sm_mhz") or float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
                                             .get("clocks_under_load", {}).get("sm_mhz_median", 1417.0))
     sms = torch.cuda.get_device_properties(local).multi_processor_count
-    peak_tops = sms * ALU_LANES_PER_SM * sm_mhz * 1e6 / 1e12
+    nominal_tops = sms * ALU_LANES_PER_SM * sm_mhz * 1e6 / 1e12
+    probe_sampler = ClockSampler(uuid)
+    time.sleep(0.3)
+    peaks = probe_peaks(sim, stream)
+    probe_clocks = probe_sampler.stop()
+    peak_tops = peaks["add"]
+    # the event-driven kernel's own algorithmic work, counted from the outputs
+    # of one sweep (starts and completions per request, distinct event steps)
+    res = S.sweep(a, p, o, policies, deltas, kv, per_request=True, counts=cnt, slack=slk)
+    st_h, co_h = res["start"], res["completion"]
+    n_events = int((st_h >= 0).sum() + (co_h >= 0).sum())
+    n_epochs = epoch_count(st_h, co_h)
+    del res, st_h, co_h
+    ops_step = OPS_PER_TOKEN_ADVANCE * tok_per_step + OPS_PER_BATCH_STEP * busy_per_step
+    ops_epoch = OPS_PER_REQUEST_EVENT * n_events + OPS_PER_EPOCH * n_epochs
+
+    def roof(kernel_name, ops, ms_per_launch, traffic):
+        achieved = ops / (ms_per_launch / 1e3) / 1e12
+        return {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s",
+                "frac": achieved / peak_tops, "traffic": traffic, "kernel": kernel_name,
+                "ops_per_launch": ops, "sim_ms_per_launch": ms_per_launch,
+                "peak_measured": peaks["add"], "alu_pipe_peak_measured": peaks["minmax"],
+                "frac_of_alu_pipe": achieved / peaks["minmax"], "peak_nominal": nominal_tops,
+                "peak_basis": (f"measured: isjl_probe_int_rate, int32 add chains ({peaks['add']:.2f} Tops/s) and "
+                               f"min/max chains ({peaks['minmax']:.2f} Tops/s), best of {PROBE_LAUNCHES} "
+                               f"full-occupancy launches at {probe_clocks.get('sm_mhz')} MHz; nominal "
+                               f"{sms} SMs x {ALU_LANES_PER_SM} lanes x {sm_mhz:.0f} MHz = {nominal_tops:.2f}")}
+
+    full = wid == DEFAULT_WID and n_inst == wl.n_instances
+    sim_avg_ms = sum(sim_ms) / len(sim_ms)
     if epoch:
-        roofline = {"bound": "alu", "achieved": None, "peak": peak_tops, "unit": "Tops/s", "frac": None,
-                    "traffic": None, "kernel": "sim_kernel (epoch)",
-                    "note": "event-driven kernel: per-token work is replaced by closed forms; see the step kernel"}
+        roofline = roof("sim_kernel (epoch)", ops_epoch, sim_avg_ms, None)
     else:
-        ops = OPS_PER_TOKEN_ADVANCE * tok_per_step + OPS_PER_BATCH_STEP * busy_per_step
-        achieved = ops / (sim_avg_ms / 1e3) / 1e12
-        full = wid == DEFAULT_WID and n_inst == wl.n_instances
-        roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s",
-                    "frac": achieved / peak_tops,
-                    "traffic": SIM_DRAM_BYTES_PER_LAUNCH if full else None,
-                    "kernel": "sim_kernel (step)", "ops_per_launch": ops,
-                    "peak_basis": f"{sms} SMs x {ALU_LANES_PER_SM} int32 lanes x {sm_mhz:.0f} MHz (median SM clock "
-                                  "sampled during the timed steps)",
-                    "sim_ms_per_launch": sim_avg_ms}
+        roofline = roof("sim_kernel (step)", ops_step, sim_avg_ms, SIM_DRAM_BYTES_PER_LAUNCH if full else None)
+    if other is not None:
+        o_ops = ops_epoch if other["kernel"] == "epoch" else ops_step
+        o_roof = roof(f"sim_kernel ({other['kernel']})", o_ops, other["sim_ms_per_launch"], None)
+        other["roofline"] = {k: o_roof[k] for k in ("achieved", "frac", "frac_of_alu_pipe", "ops_per_launch")}
+        other["epochs_per_launch"] = n_epochs
+        other["request_events_per_launch"] = n_events
 
     cpu = None
     if pool is not None:
@@ -420,10 +483,13 @@ def main():
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": ({"value": units_all / (e2e_ms_all / 1e3) / args.steps, "unit": UNIT,
-                 "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"]} if e2e else None),
+                 "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"],
+                 "outputs": "records only: the host entry point returns the per-(run, instance) records; "
+                            "per-request start / completion steps are not copied back"} if e2e else None),
         "gpu_launches": launches_per_step * args.steps,
         "clocks": {"sm_mhz": clocks.get("sm_mhz"), "sm_max_mhz": clocks.get("sm_max_mhz"),
-                   "reasons": clocks.get("reasons")},
+                   "reasons": clocks.get("reasons"), "probe_sm_mhz": probe_clocks.get("sm_mhz"),
+                   "probe_reasons": probe_clocks.get("reasons")},
         "instances_per_s": world * n_inst * len(policies) * args.steps / (t_ms_all / 1e3),
         "token_advances_per_s": tok_per_step * world * args.steps / (t_ms_all / 1e3),
         "kernel_ms": {"sim": sim_avg_ms},

@@ -92,7 +92,9 @@ typedef struct {
 typedef struct {
     const int32_t *arrival;  /* release step A_i >= 0, non-decreasing within an instance */
     const int32_t *prompt;   /* prompt tokens >= 0 */
-    const int32_t *output;   /* output tokens >= 0; o_i = prompt + output must be 1..ISJL_MAX_LEN */
+    const int32_t *output;   /* output tokens >= 0; o_i = prompt + output must be 1..ISJL_MAX_LEN, and
+                                per instance sum o_i + max A_i <= 2^30 - 2 (the range of the step
+                                counter); an instance beyond either limit is INVALID_ARG */
     const int32_t *count;    /* device, n_instances entries or NULL: instance i uses its first
                                 count[i] slots (0..n_per_instance; 0 = an empty instance, all
                                 counters 0); NULL = every instance uses all n_per_instance.  A
@@ -209,7 +211,8 @@ isjl_status isjl_sim_run_sweep_host(isjl_sim *sim, int32_t n_runs, const int32_t
 /* Wait for the last run/sweep on its stream and copy its per-run summaries
  * into the host array out (capacity max_runs >= the last call's n_runs).
  * Returns the first nonzero device status of the last call (INFEASIBLE,
- * INVALID_ARG, STEP_LIMIT), NOT_READY if nothing ran, CUDA on a failed sync. */
+ * INVALID_ARG, STEP_LIMIT, INTERNAL), NOT_READY if nothing ran, CUDA on a
+ * failed sync. */
 isjl_status isjl_sim_metrics(isjl_sim *sim, isjl_summary *out, int32_t max_runs);
 
 /* Number of kernels the last run/sweep call launched (0 if none). */
@@ -244,15 +247,29 @@ int32_t isjl_sim_kernel_times(const isjl_sim *sim, float *ms, int32_t cap);
  * serialized by the caller.  Asynchronous on stream.
  *
  * Limit: the workspace needs 16 bytes per request (20 when
- * n_per_instance > 4096), 40 bytes per instance, and n_per_instance * 16 bytes
- * per block of the simulation kernel; fewer blocks run when the array cannot
- * hold all resident ones.  That is about 3 to 4 million requests per call.
+ * n_per_instance > 4096, and 4 more when in->slack is given, for the true
+ * lengths), 40 bytes per instance, and n_per_instance * 16 bytes per block of
+ * the simulation kernel; fewer blocks run when the array cannot hold all
+ * resident ones.  That is about 3 to 4 million requests per call.
  * Errors: INVALID_ARG (as isjl_sim_run_sweep, or the problem does not fit the
  * fixed workspace), CUDA (symbol lookup or launch failure). */
 #define ISJL_NOALLOC_SCRATCH_BYTES (64u << 20)
 isjl_status isjl_sim_run_sweep_noalloc(const isjl_config *cfg, int32_t n_runs, const int32_t *policies,
                                        const int32_t *deltas, int32_t kv_cap, const isjl_instances *in,
                                        const isjl_outputs *out, void *stream);
+
+/* Measurement helper; the paper has no counterpart.  The rate at which the
+ * current GPU executes simple int32 instructions: the denominator of the
+ * simulation kernels' roofline (they are bound by integer issue, not by memory
+ * or tensor throughput).  kind 0: 32-bit adds; kind 1: 32-bit min / max (the
+ * instructions of a step's extent).  One launch on stream that fills every SM
+ * (256-thread blocks, as many per SM as fit), each thread running
+ * iters x 128 instructions spread over 8 independent dependency chains; waits
+ * for it.  Writes, to host memory, the int32 lane-instructions executed
+ * (threads x iters x 128) to *lane_instructions and the launch's CUDA-event
+ * time in milliseconds to *ms.  Errors: INVALID_ARG (kind not 0 or 1,
+ * iters < 1, a null pointer), CUDA. */
+isjl_status isjl_probe_int_rate(int32_t kind, int32_t iters, void *stream, double *lane_instructions, float *ms);
 
 /* Static description of a status code (never NULL). */
 const char *isjl_status_string(isjl_status status);

@@ -63,7 +63,7 @@ assert ctypes.sizeof(isjl_record) == RECORD_DTYPE.itemsize == 192
 
 EXPORTS = ["isjl_sim_create", "isjl_sim_destroy", "isjl_sim_run", "isjl_sim_run_sweep",
            "isjl_sim_run_sweep_host", "isjl_sim_metrics", "isjl_sim_last_launches", "isjl_sim_kernel_times",
-           "isjl_sim_run_sweep_noalloc", "isjl_status_string"]
+           "isjl_sim_run_sweep_noalloc", "isjl_probe_int_rate", "isjl_status_string"]
 
 _lib = None
 
@@ -97,6 +97,9 @@ def lib():
         L.isjl_sim_run_sweep_noalloc.argtypes = [ctypes.POINTER(isjl_config), i32, p32, p32, i32,
                                                  ctypes.POINTER(isjl_instances), ctypes.POINTER(isjl_outputs), vp]
         L.isjl_sim_run_sweep_noalloc.restype = ctypes.c_int
+        L.isjl_probe_int_rate.argtypes = [i32, i32, vp, ctypes.POINTER(ctypes.c_double),
+                                          ctypes.POINTER(ctypes.c_float)]
+        L.isjl_probe_int_rate.restype = ctypes.c_int
         L.isjl_status_string.argtypes = [ctypes.c_int]
         L.isjl_status_string.restype = ctypes.c_char_p
         _lib = L
@@ -128,6 +131,16 @@ def _policy_code(p):
 
 
 # ---- thin wrappers with the C names ----------------------------------------
+def isjl_probe_int_rate(kind, iters, stream=None):
+    """(int32 lane-instructions executed, milliseconds) of one probe launch;
+    kind 0 = adds, 1 = min / max."""
+    n = ctypes.c_double()
+    ms = ctypes.c_float()
+    _check(lib().isjl_probe_int_rate(int(kind), int(iters), _stream_ptr(stream), ctypes.byref(n), ctypes.byref(ms)),
+           "isjl_probe_int_rate")
+    return n.value, ms.value
+
+
 def isjl_sim_create(n_instances, n_per_instance, B, c=0.0005, tau=1e-6, p0=0.002, max_steps=0,
                     flags=FLAG_STEP_KERNEL):
     cfg = isjl_config(int(n_instances), int(n_per_instance), int(B), float(c), float(tau), float(p0),

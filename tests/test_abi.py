@@ -41,6 +41,17 @@ def test_binding_loads_and_status_strings(built_lib):
     assert "step limit" in sim.isjl_status_string(5)
 
 
+def test_probe_rejects_bad_arguments_without_a_gpu(built_lib):
+    """Argument checks come before any CUDA call."""
+    from paper_2608_02244_gb300 import sim
+    n, ms = ctypes.c_double(), ctypes.c_float()
+    L = sim.lib()
+    assert L.isjl_probe_int_rate(2, 10, None, ctypes.byref(n), ctypes.byref(ms)) == sim.ISJL_ERR_INVALID_ARG
+    assert L.isjl_probe_int_rate(0, 0, None, ctypes.byref(n), ctypes.byref(ms)) == sim.ISJL_ERR_INVALID_ARG
+    assert L.isjl_probe_int_rate(1, 10, None, None, ctypes.byref(ms)) == sim.ISJL_ERR_INVALID_ARG
+    assert "internal" in sim.isjl_status_string(sim.ISJL_ERR_INTERNAL)
+
+
 def test_ctypes_layout_matches_header():
     """Compile the header with gcc and compare sizes/offsets with the binding."""
     from paper_2608_02244_gb300 import sim

@@ -48,6 +48,7 @@ def run_both(S, O, a, p, o, B, policies, deltas, kv, epoch, per_request=True, ma
     finally:
         sm.close()
     assert res["launches"] == 4
+    assert (res["records"]["status"] != S.ISJL_ERR_INTERNAL).all()   # no kernel invariant ever fails
     if check:
         for i, (pol, d) in enumerate(zip(policies, deltas)):
             rec, st, co = O.run(pol, B, d, kv, a, p, o, max_steps=max_steps, per_request=per_request,
@@ -320,6 +321,51 @@ def test_bulk_starts_with_ties_and_partial_rows(S, O, epoch):
     for B in (33, 100, 256):
         for kv in (INF, 700):
             run_both(S, O, a, p, o, B, pols, ds, kv, epoch)
+
+
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_domain_limits(S, O, epoch):
+    """The GPU's documented limits, against the oracle just below them: a
+    request of ISJL_MAX_LEN = 65,535 tokens, and an instance whose
+    sum o + max arrival is 2^30 - 2 (the step counter's range), run and agree
+    with the oracle; one token more at either limit is INVALID_ARG on the GPU
+    (the oracle has no such limit and simulates it)."""
+    # o_i = 65,535 next to short requests, with arrivals
+    a = np.array([[0, 0, 3, 9]], np.int32)
+    p = np.array([[65000, 3, 0, 7]], np.int32)
+    o = np.array([[535, 4, 11, 2]], np.int32)
+    run_both(S, O, a, p, o, 2, ["fcfs", "ljf", "isjl", "sjf"], [0, 0, 6, 0], INF, epoch)
+    o2 = o.copy()
+    o2[0, 0] += 1                                   # 65,536 tokens
+    res = run_both(S, O, a, p, o2, 2, ["fcfs"], [0], INF, epoch, check=False)
+    assert res["records"][0]["status"][0] == S.ISJL_ERR_INVALID_ARG
+    # sum o + max arrival = 2^30 - 2: 16,384 requests of 65,535 tokens and one of 16,382
+    n = 16_385
+    a = np.zeros((1, n), np.int32)
+    p = np.full((1, n), 65_000, np.int32)
+    o = np.full((1, n), 535, np.int32)
+    p[0, -1] = 0                                    # the last request: 16,382 tokens in all
+    o[0, -1] = 16_382
+    assert int((p + o).astype(np.int64).sum()) == 2**30 - 2
+    run_both(S, O, a, p, o, 512, ["fcfs", "ljf"], [0, 0], INF, epoch, per_request=False)
+    o3 = o.copy()
+    o3[0, -1] += 1                                  # sum o + max arrival = 2^30 - 1
+    res = run_both(S, O, a, p, o3, 512, ["fcfs"], [0], INF, epoch, per_request=False, check=False)
+    assert res["records"][0]["status"][0] == S.ISJL_ERR_INVALID_ARG
+
+
+def test_integer_rate_probe(S):
+    """The roofline denominators: both probe kinds run, count their
+    instructions and report a rate within what 152 SMs can issue."""
+    import torch
+    for kind in (0, 1):
+        n, ms = S.isjl_probe_int_rate(kind, 200)
+        props = torch.cuda.get_device_properties(0)
+        blocks = n / (256 * 200 * 128)          # one full wave: a whole number of blocks per SM
+        assert blocks == int(blocks) and int(blocks) % props.multi_processor_count == 0
+        rate = n / (ms / 1e3)
+        # at most 128 lanes per SM at 2.2 GHz, and surely more than 1 Tops/s
+        assert 1e12 < rate < props.multi_processor_count * 128 * 2.2e9, (kind, rate)
 
 
 def test_invalid_arguments_rejected(S):
