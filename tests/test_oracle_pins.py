@@ -291,3 +291,103 @@ def test_oracle_errors(oracle_mod):
     assert oracle_mod.run("fcfs", 2, 0, INF, z, np.array([0, -1, 0], np.int32), o)[0]["status"] == 1
     assert oracle_mod.run("fcfs", 0, 0, INF, z, z, o)[0]["status"] == 1
     assert oracle_mod.run("isjl", 2, 0, INF, z, z, o, max_steps=2)[0]["status"] == 5
+
+
+@pytest.mark.parametrize("policy", ["isjl", "isjl_beta"])
+def test_b2_first_stage_follows_the_stage_definition(oracle_mod, policy):
+    """B = 2, all requests at t = 0, o_2 > alpha: the first stage is the one
+    the proof of Theorem "Competitive ratio of Algorithm ISJL" defines (its
+    "stage" definition): the pack P runs alone for P - alpha steps (if
+    positive), L = o_1 joins it until P ends, then S = o_2 starts beside L.
+    The pack is the B = 2 rule of Section 3.2: scanning the shorter requests
+    longest first, take each that keeps the pack within
+    q = min{o_1 - o_2 + beta, 2 alpha} (beta = alpha for Algorithm 2)."""
+    O = oracle_mod
+    rng = np.random.default_rng(31 if policy == "isjl" else 32)
+    checked = 0
+    for _ in range(400):
+        n = int(rng.integers(3, 12))
+        o = rng.integers(1, 60, n).astype(np.int32)
+        alpha = int(rng.integers(1, 30))
+        order = sorted(range(n), key=lambda i: (-int(o[i]), i))
+        o1, o2 = int(o[order[0]]), int(o[order[1]])
+        if o2 <= alpha:
+            continue
+        beta = alpha if policy == "isjl" else O.beta(alpha)
+        q = min(o1 - o2 + beta, 2 * alpha)
+        pack, P = [], 0
+        for i in order[2:]:
+            if P + int(o[i]) <= q:
+                pack.append(i)
+                P += int(o[i])
+        _, st, co = O.run(policy, 2, alpha, INF, np.zeros(n, np.int32), np.zeros(n, np.int32), o)
+        t = 0
+        for i in pack:                     # the pack runs back to back from step 0
+            assert st[i] == t, (o, alpha, pack)
+            t += int(o[i])
+        assert st[order[0]] == max(P - alpha, 0)     # L joins after P - alpha steps
+        assert st[order[1]] == P                     # S starts when the pack ends
+        # Phase TWO at the first freed worker (Section 3.2): the longest
+        # unprocessed request starts there if the other worker's decode length
+        # is at most alpha, else not before the other one ends
+        endL, endS = int(co[order[0]]), int(co[order[1]])
+        rest = [i for i in order[2:] if i not in pack]
+        if rest and endL != endS:
+            t1, other_start, other_end = ((endL, P, endS) if endL < endS else (endS, st[order[0]], endL))
+            nxt = rest[0]
+            if t1 - other_start <= alpha:
+                assert st[nxt] == t1, (o, alpha)
+            else:
+                assert st[nxt] >= other_end, (o, alpha)
+        checked += 1
+    assert checked > 100
+
+
+@pytest.mark.parametrize("B", [3, 4, 6])
+def test_first_stage_timing_with_short_packs(oracle_mod, B):
+    """B >= 3, all requests at t = 0, at most B requests longer than alpha and
+    the rest at most alpha long: Algorithm 2's first stage as Section 3.3
+    describes it.  Each pack runs back to back from step 0 on its worker (a
+    pack member of length <= alpha can never shut the gate), o_1 is held back
+    d1 = min{max{max_j sum(w_j) - alpha, 0}, alpha} steps, and each long
+    request o_j (2 <= j <= M) starts on its worker when its pack has ended,
+    and not before o_1.  Packs: each shorter request, longest first, goes to
+    the first worker with room, visiting the workers without a long request
+    (budget alpha) in order, then the workers of o_M, ..., o_2 (budget
+    min{2 alpha, o_1 - o_j + alpha})."""
+    O = oracle_mod
+    rng = np.random.default_rng(40 + B)
+    checked = 0
+    for _ in range(300):
+        alpha = int(rng.integers(2, 25))
+        n_long = int(rng.integers(2, B + 1))
+        n_short = int(rng.integers(0, 3 * B))
+        o = np.concatenate([rng.integers(alpha + 1, 4 * alpha + 2, n_long),
+                            rng.integers(1, alpha + 1, n_short)]).astype(np.int32)
+        o = o[rng.permutation(len(o))]
+        n = len(o)
+        order = sorted(range(n), key=lambda i: (-int(o[i]), i))
+        M = n_long
+        o1 = int(o[order[0]])
+        budget = {j: alpha for j in range(M + 1, B + 1)}
+        budget.update({j: min(2 * alpha, o1 - int(o[order[j - 1]]) + alpha) for j in range(2, M + 1)})
+        visit = list(range(M + 1, B + 1)) + list(range(M, 1, -1))
+        packs = {j: [] for j in visit}
+        for i in order[M:]:
+            for j in visit:
+                if sum(int(o[x]) for x in packs[j]) + int(o[i]) <= budget[j]:
+                    packs[j].append(i)
+                    break
+        sums = {j: sum(int(o[x]) for x in packs[j]) for j in visit}
+        d1 = min(max(max(sums[j] for j in range(2, M + 1)) - alpha, 0), alpha)
+        _, st, _ = O.run("isjl", B, alpha, INF, np.zeros(n, np.int32), np.zeros(n, np.int32), o)
+        for j in visit:
+            t = 0
+            for i in packs[j]:
+                assert st[i] == t, (o.tolist(), alpha, j)
+                t += int(o[i])
+        assert st[order[0]] == d1, (o.tolist(), alpha)
+        for j in range(2, M + 1):
+            assert st[order[j - 1]] == max(sums[j], d1), (o.tolist(), alpha, j)
+        checked += 1
+    assert checked == 300
