@@ -13,9 +13,12 @@
 // Layout.  Worker (batch slot) w lives in lane w % 32, register row w / 32,
 // so a warp holds B <= 32 * SPL workers.  The step kernel advances, each
 // step, every slot of the rows that hold a running worker (a per-row-count
-// instantiation of the step loop), straight-line: an idle slot carries a
-// progress below 0 as a signed value and at least 2^31 as an unsigned one, so
-// the step's max (signed) and min (unsigned) need no per-slot predicate.  The
+// instantiation of the step loop), straight-line: from 8 rows on, a slot's
+// progress a is packed as (a << 16) | (65535 - a), so one add advances it and
+// one per-half max collects both the step's max and (complemented) min, with
+// idle slots set at the start of each stretch to values that lose both;
+// below 8 rows an idle slot carries a progress below 0 as a signed value and
+// at least 2^31 as an unsigned one (signed max, unsigned min).  The
 // sum of progress over all steps is added per request, o (o + 1) / 2, when it
 // starts (a run stopped early takes back the unserved part).  Values that
 // change only at events (next
@@ -49,7 +52,11 @@ namespace isjl {
 namespace {
 
 constexpr int32_t kNone = -1;
-constexpr int32_t kIdle = -(1 << 30);   // idle-slot progress sentinel base
+constexpr int32_t kIdle = -(1 << 30);   // idle-slot progress sentinel base (unpacked step kernel)
+// step kernel with SPL >= 8: the progress a of a slot is packed as
+// (a << 16) | (65535 - a)
+constexpr uint32_t kPackedZero = 0xFFFFu;  // a = 0
+constexpr uint32_t kPackedStep = 0xFFFFu;  // one step: a + 1 above, 65535 - (a + 1) below
 
 struct WarpSmem {
     int32_t *sjob;    // [B] request running on worker w
@@ -130,6 +137,13 @@ __device__ __forceinline__ void dispatch_rows(int rows, F &f) {
         if (rows <= C::at(MID)) dispatch_rows<SPL, LO, MID>(rows, f);
         else dispatch_rows<SPL, MID + 1, HI>(rows, f);
     }
+}
+
+// per-16-bit-half unsigned maximum
+__device__ __forceinline__ uint32_t vmax_u16x2(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("max.u16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
 }
 
 // acc += a * b into a 64-bit accumulator with one wide multiply-add
@@ -265,6 +279,10 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     int32_t *st_out = A.start_out ? A.start_out + out_off : nullptr;
     int32_t *co_out = A.compl_out ? A.compl_out + out_off : nullptr;
     const int words0 = (n + 31) >> 5, words1 = (words0 + 31) >> 5;
+    // packed progress in the step kernel's stretch pays off from 8 register
+    // rows on (measured); fewer rows keep the signed / unsigned sentinel
+    constexpr bool kPacked = !EPOCH && SPL >= 8;
+    constexpr int32_t kStartA = EPOCH ? 0 : (kPacked ? (int32_t)kPackedZero : 0);
 
     int64_t status = is.status;
     if (status == ISJL_OK && (int64_t)is.maxo > kv_cap) status = ISJL_ERR_INFEASIBLE;
@@ -362,7 +380,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (lane == owner) {
 #pragma unroll
                 for (int r = 0; r < SPL; ++r)
-                    if (r == row) { sa[r] = EPOCH ? k : 0; sc[r] = k + oc; }
+                    if (r == row) { sa[r] = EPOCH ? k : kStartA; sc[r] = k + oc; }
                 busy |= 1u << row;
                 lane_cmin = min(lane_cmin, k + oc);
                 S.sres[w] = oe;
@@ -429,7 +447,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     const int oc = __shfl_sync(kFull, oc_l, src);
                     if (f && rank < c) {
                         const int w = (r << 5) + lane;
-                        sa[r] = EPOCH ? k : 0;
+                        sa[r] = EPOCH ? k : kStartA;
                         sc[r] = k + oc;
                         busy |= 1u << r;
                         my_cmin = min(my_cmin, k + oc);
@@ -456,7 +474,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (f) {
                     if (EPOCH) sf += (unsigned)(sa[r] - (c - 65536));
                     sc[r] = INT_MAX;
-                    if (!EPOCH) sa[r] = kIdle;
+                    if (!EPOCH && !kPacked) sa[r] = kIdle;
                 }
             }
             // per finishing request (usually one per warp): outputs and its KV release
@@ -493,10 +511,17 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             if (run_cnt == 0) return 0;
             if (EPOCH) return (int64_t)k - smin;
             if (!amax_ok) {
-                int m = 0;
+                if constexpr (kPacked) {
+                    uint32_t m = 0u;    // packed progress: the larger value has the larger a
 #pragma unroll
-                for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = max(m, sa[r]);
-                amax_c = __reduce_max_sync(kFull, m);
+                    for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = max(m, (uint32_t)sa[r]);
+                    amax_c = (int32_t)(__reduce_max_sync(kFull, m) >> 16);
+                } else {
+                    int m = 0;
+#pragma unroll
+                    for (int r = 0; r < SPL; ++r) if (busy >> r & 1u) m = max(m, sa[r]);
+                    amax_c = __reduce_max_sync(kFull, m);
+                }
                 amax_ok = true;
             }
             return amax_c;
@@ -655,7 +680,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         if (w >= 1 && w < nlong && nx >= 0 && nx == S.slong[w]) lhead |= bit;
                         else lhead &= ~bit;
                         const int oc = otru ? otru[e] : oe;     // it finishes after its true length
-                        sa[r] = EPOCH ? k : 0;
+                        sa[r] = EPOCH ? k : kStartA;
                         sc[r] = k + oc;
                         busy |= bit;
                         my_cmin = min(my_cmin, k + oc);
@@ -964,35 +989,70 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         };
 
         // steps k .. k + L - 1 with no event: advance rows [0, NR), which hold
-        // every running worker, and add each step's cost (max r and min r by
-        // warp reductions; idle slots hold a value below 0 as a signed number
-        // and at least 2^31 as an unsigned one, so they lose both)
+        // every running worker, and add each step's cost.
+        //   SPL >= 8: a slot's progress a is packed as (a << 16) | (65535 - a)
+        //   (o <= 65535): one add of 0xFFFF advances both halves (no borrow: a < o
+        //   while the request runs), and a per-half unsigned max over a lane's
+        //   slots, then two warp max reductions, give max r (upper half) and
+        //   65535 - min r (lower half).  Idle slots of these rows are first set
+        //   to (0, L): after j steps they hold (j, L - j), at most the running
+        //   slots' halves, since every running request has a >= j and none
+        //   completes inside the stretch (min a + L <= its o <= 65535).
+        //   SPL < 8: idle slots hold a value below 0 as a signed number and at
+        //   least 2^31 as an unsigned one, so they lose the signed max and the
+        //   unsigned min.
         auto plain_steps = [&](auto nr_tag, int L) {
             constexpr int NR = decltype(nr_tag)::value;
             const uint32_t cnt = (uint32_t)run_cnt;
-            int last_mx = 0;
             constexpr int kUnroll = SPL >= 16 ? 4 : 2;   // measured; more code costs instruction-cache misses
-#pragma unroll kUnroll
-            for (int j = 0; j < L; ++j) {
-                int mx = INT_MIN;
-                unsigned mn = 0xffffffffu;
+            if constexpr (kPacked) {
 #pragma unroll
-                for (int r = 0; r < NR; ++r) {
-                    const int a = sa[r] + 1;
-                    sa[r] = a;
-                    mx = max(mx, a);
-                    mn = min(mn, (unsigned)a);
+                for (int r = 0; r < NR; ++r)
+                    if (!(busy >> r & 1u)) sa[r] = L;
+                uint32_t last_mx = 0u;
+#pragma unroll kUnroll
+                for (int j = 0; j < L; ++j) {
+                    uint32_t m = 0u;
+#pragma unroll
+                    for (int r = 0; r < NR; ++r) {
+                        const uint32_t a = (uint32_t)sa[r] + kPackedStep;
+                        sa[r] = (int32_t)a;
+                        m = vmax_u16x2(m, a);
+                    }
+                    const uint32_t mx = __reduce_max_sync(kFull, m) >> 16;          // max r
+                    const uint32_t lo = __reduce_max_sync(kFull, m & 0xFFFFu);      // 65535 - min r
+                    const int ext = (int)(mx + lo) - 65535;
+                    mad_wide(W, cnt, mx);                // |S| max r
+                    mad_wide(sumext, (uint32_t)ext, 1u);
+                    maxext = max(maxext, ext);
+                    viol += ext > alpha32;
+                    last_mx = mx;
                 }
-                mx = __reduce_max_sync(kFull, mx);
-                mn = __reduce_min_sync(kFull, mn);
-                const int ext = mx - (int)mn;
-                mad_wide(W, cnt, (uint32_t)mx);      // |S| max r
-                mad_wide(sumext, (uint32_t)ext, 1u);
-                maxext = max(maxext, ext);
-                viol += ext > alpha32;
-                last_mx = mx;
+                amax_c = (int32_t)last_mx;               // max progress entering step k + L
+            } else {
+                int last_mx = 0;
+#pragma unroll kUnroll
+                for (int j = 0; j < L; ++j) {
+                    int mx = INT_MIN;
+                    unsigned mn = 0xffffffffu;
+#pragma unroll
+                    for (int r = 0; r < NR; ++r) {
+                        const int a = sa[r] + 1;
+                        sa[r] = a;
+                        mx = max(mx, a);
+                        mn = min(mn, (unsigned)a);
+                    }
+                    mx = __reduce_max_sync(kFull, mx);
+                    mn = __reduce_min_sync(kFull, mn);
+                    const int ext = mx - (int)mn;
+                    mad_wide(W, cnt, (uint32_t)mx);      // |S| max r
+                    mad_wide(sumext, (uint32_t)ext, 1u);
+                    maxext = max(maxext, ext);
+                    viol += ext > alpha32;
+                    last_mx = mx;
+                }
+                amax_c = last_mx;                        // max progress entering step k + L
             }
-            amax_c = last_mx;                        // max progress entering step k + L
             amax_ok = true;
         };
 
@@ -1036,7 +1096,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 #pragma unroll
             for (int r = 0; r < SPL; ++r)
                 if (busy >> r & 1u) {
-                    const uint32_t a = (uint32_t)sa[r], o = a + (uint32_t)(sc[r] - k);
+                    const uint32_t a = kPacked ? (uint32_t)sa[r] >> 16 : (uint32_t)sa[r];
+                    const uint32_t o = a + (uint32_t)(sc[r] - k);
                     unserved += (int64_t)((o * (o + 1u)) >> 1) - (int64_t)((a * (a + 1u)) >> 1);
                 }
             E = W - (R - warp_sum64(unserved));

@@ -59,6 +59,44 @@ def test_noalloc_matches_regular_sweep_twice(epoch):
             np.testing.assert_array_equal(co.cpu().numpy().reshape(len(pols), n_inst, n), want["completion"])
 
 
+@pytest.mark.parametrize("epoch", [False, True])
+def test_noalloc_fewer_blocks_and_slack(epoch):
+    """Large instances (n = 100,000): the fixed array holds the plan scratch of
+    fewer simulation blocks than are resident, so the call runs on fewer
+    warps; and a robust workload, whose true lengths take 4 more bytes per
+    request.  Both must match the regular sweep, records and per-request steps."""
+    import torch
+    from paper_2608_02244_gb300 import sim, workloads as W
+    flags = sim.FLAG_EPOCH_KERNEL if epoch else sim.FLAG_STEP_KERNEL
+    cases = [(5, 3, 512, 1_000_000, ["fcfs", "isjl"], [0, 256], False),
+             (8, 12, 256, 200_000, ["fcfs", "ljf", "isjl", "isjl"], [0, 0, 64, INF], True)]
+    for wid, count, B, kv, pols, ds, robust in cases:
+        a_h, p_h, o_h, _, e_h = W.generate(wid, count, with_counts=True, with_slack=True)
+        e_h = e_h if robust else None
+        n_inst, n = a_h.shape
+        if wid == 5:   # the plan scratch of the resident blocks does not fit: fewer blocks run
+            free = (64 << 20) - n_inst * n * 20 - 4096
+            assert free // (4 * n) < 4 * 152
+        ref = sim.Simulator(n_inst, n, B, epoch=epoch)
+        try:
+            want = ref.sweep(a_h, p_h, o_h, pols, ds, kv, per_request=True, slack=e_h)
+        finally:
+            ref.close()
+        a, p, o = (torch.from_numpy(x).cuda() for x in (a_h, p_h, o_h))
+        e = torch.from_numpy(e_h).cuda() if e_h is not None else None
+        rec = torch.zeros(len(pols) * n_inst * sim.RECORD_DTYPE.itemsize, dtype=torch.uint8, device="cuda")
+        st = torch.full((len(pols) * n_inst * n,), -7, dtype=torch.int32, device="cuda")
+        co = torch.full_like(st, -7)
+        rc = sim.isjl_sim_run_sweep_noalloc(n_inst, n, B, pols, ds, kv, a, p, o, rec, st, co, flags=flags, slack=e)
+        assert rc == sim.ISJL_OK, sim.isjl_status_string(rc)
+        torch.cuda.synchronize()
+        got = sim.records_to_numpy(rec, len(pols), n_inst)
+        for i in range(len(pols)):
+            _check_equal(got[i], want["records"][i])
+        np.testing.assert_array_equal(st.cpu().numpy().reshape(len(pols), n_inst, n), want["start"])
+        np.testing.assert_array_equal(co.cpu().numpy().reshape(len(pols), n_inst, n), want["completion"])
+
+
 def test_noalloc_rejects_oversize_problem():
     import torch
     from paper_2608_02244_gb300 import sim
