@@ -1056,6 +1056,75 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             amax_ok = true;
         };
 
+        // epoch kernel: the step at which the running set's earliest or latest
+        // start changes (the last completion among the requests that started at
+        // smin, or at smax)
+        auto window_end = [&]() -> int32_t {
+            int32_t e_lo = INT_MIN, e_hi = INT_MIN;
+#pragma unroll
+            for (int r = 0; r < SPL; ++r)
+                if (busy >> r & 1u) {
+                    if (sa[r] == smin) e_lo = max(e_lo, sc[r]);
+                    if (sa[r] == smax) e_hi = max(e_hi, sc[r]);
+                }
+            return min(__reduce_max_sync(kFull, e_lo), __reduce_max_sync(kFull, e_hi));
+        };
+        // epoch kernel: serve steps k .. K - 1 at once, K <= the step at which
+        // the earliest or latest start changes.  Every running request i
+        // (start s_i, completion c_i) runs L_i = min(c_i, K) - k of them, with
+        // max r = t - smin + 1 at step t and r_i = t - s_i + 1:
+        //   W += L_i (k - smin + 1) + L_i (L_i - 1) / 2,  E += L_i (s_i - smin),
+        // and the extent smax - smin is constant.  Requests with c_i < K
+        // complete inside the window and leave here.
+        auto window = [&](int32_t K) {
+            const int64_t m0 = (int64_t)k - smin + 1;
+            int64_t wl = 0, el = 0, cl = 0, sl = 0;
+            int32_t tl = 0, cmx = 0, nf = 0, of = 0;
+            uint32_t fm = 0u;
+#pragma unroll
+            for (int r = 0; r < SPL; ++r)
+                if (busy >> r & 1u) {
+                    const int32_t c = sc[r];
+                    const int64_t Li = (int64_t)min(c, K) - k;
+                    wl += Li * m0 + Li * (Li - 1) / 2;
+                    el += Li * (int64_t)(sa[r] - smin);
+                    tl += (int32_t)Li;
+                    if (c < K) {                                  // completes inside the window
+                        const int w = (r << 5) + lane;
+                        fm |= 1u << r;
+                        cl += c;
+                        sl += sa[r];
+                        cmx = max(cmx, c);
+                        nf++;
+                        of += S.sres[w];
+                        if (co_out) co_out[S.sjob[w]] = c;
+                        sc[r] = INT_MAX;
+                    }
+                }
+            busy &= ~fm;
+            recompute_lane();
+            W += warp_sum64(wl);
+            E += warp_sum64(el);
+            tok += (int32_t)__reduce_add_sync(kFull, (unsigned)tl);
+            nf = (int32_t)__reduce_add_sync(kFull, (unsigned)nf);
+            of = (int32_t)__reduce_add_sync(kFull, (unsigned)of);
+            sumc += warp_sum64(cl);
+            sum_st -= warp_sum64(sl);
+            const int32_t cm = (int32_t)__reduce_max_sync(kFull, (unsigned)cmx);
+            if (nf > 0) Tmake = max(Tmake, cm);
+            done += nf;
+            run_cnt -= nf;
+            kv_sum -= of;
+            kv_over = kv_sum > kv_cap;
+            cmin = __reduce_min_sync(kFull, lane_cmin);
+            const int32_t ext = smax - smin;                  // unchanged inside the window
+            const int32_t L = K - k;
+            sumext += (int64_t)L * ext;
+            maxext = max(maxext, ext);
+            viol += ext > alpha32 ? L : 0;
+            Tb += L;
+        };
+
         // release every request with A_i <= k (a prefix: arrivals are non-decreasing)
         if (!EPOCH) {
             // ---------------------------------------------------- step kernel
@@ -1115,6 +1184,19 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (policy == ISJL_POLICY_ISJL && !L1_started && t0 + d1 > k) nxt = min(nxt, t0 + d1);
                 if (nxt == INT_MAX) { status = ISJL_ERR_STEP_LIMIT; break; }   // cannot progress
                 nxt = min(nxt, step_guard);                          // serve no step past max_steps
+                // LJF with a batch running, or ISJL with its gate shut (A_max only
+                // grows while the earliest start stays): no request can start
+                // before the running set's earliest or latest start changes, so
+                // completions in between end no epoch of their own
+                if (run_cnt > 0 && !kv_over && nxt == cmin &&
+                    (policy == ISJL_POLICY_LJF || (policy == ISJL_POLICY_ISJL && (int64_t)k - smin > alpha))) {
+                    const int32_t K = min(window_end(), step_guard);
+                    if (K > nxt) {
+                        window(K);
+                        k = K;
+                        continue;
+                    }
+                }
                 if (run_cnt > 0) {
                     const int64_t L = nxt - k, s = run_cnt;
                     const int64_t m0 = (int64_t)k - smin + 1;       // max r at step k
