@@ -72,9 +72,9 @@ OPS_PER_EPOCH = 14
 PROBE_ITERS = 20_000
 PROBE_LAUNCHES = 3
 # DRAM bytes (read + write) per launch of the step simulation kernel on the full
-# workload: 745.0 MB measured by ncu on the first 4,096 instances, scaled by
+# workload: 748.6 MB measured by ncu on the first 4,096 instances, scaled by
 # 10,000 / 4,096 (profiles/sim_kernel_step_online_delta_sweep_4096.md)
-SIM_DRAM_BYTES_PER_LAUNCH = 745.0e6 * 10_000 / 4_096
+SIM_DRAM_BYTES_PER_LAUNCH = 748.6e6 * 10_000 / 4_096
 
 
 def workload_config(kernel, wl, n_inst, policies, deltas, flush):
