@@ -19,7 +19,7 @@
  * decomposition"): total = tau*Q + c*T + tau*E with Q = sum o(o+1)/2 and
  * E = sum over steps of sum_{i in S}(max r - r_i).
  *
- * Readings where the paper is silent (each is listed in the design notes):
+ * Readings where the paper is silent:
  *   - KV cap: a running request reserves its peak footprint o_i; a start needs
  *     sum_{S} o_j + o_i <= kv_cap.  kv_cap = INT32_MAX is the paper's model.
  *   - In every policy the first KV failure ends all starts of that step.
@@ -309,11 +309,12 @@ static int worker_free(const sim_t *s, int j) { return s->worker_job[j] < 0 && s
 static void isjl_admit(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_t *budget, int32_t *wk) {
     const int nothing_runs = (s->run_cnt == 0);
     const int64_t amax = a_max(s);
-    if (s->plan_left == 0 && longest_waiting(s, k) >= 0) {
+    const int reopen = (s->flags & V_REBUILD_REOPEN) && s->broke && !nothing_runs && amax <= s->alpha;
+    if (s->plan_left == 0 && (nothing_runs || reopen) && longest_waiting(s, k) >= 0) {
         int nw = 0;
         if (nothing_runs) {
             for (int j = 1; j <= s->B; ++j) wk[nw++] = j;
-        } else if ((s->flags & V_REBUILD_REOPEN) && s->broke && amax <= s->alpha) {
+        } else {
             for (int j = 1; j <= s->B; ++j) if (worker_free(s, j)) wk[nw++] = j;
         }
         if (nw > 0) {
@@ -355,7 +356,7 @@ static void isjl_admit(sim_t *s, int64_t k, int32_t *Q, int64_t *packsum, int64_
     }
     if (stop || !gate_ok) {
         /* a free worker and a queued request that the closed gate keeps apart */
-        if (!gate_ok && longest_waiting(s, k) >= 0)
+        if ((s->flags & V_REBUILD_REOPEN) && !gate_ok && longest_waiting(s, k) >= 0)
             for (int j = 1; j <= s->B; ++j) if (worker_free(s, j)) { s->broke = 1; break; }
         return;
     }

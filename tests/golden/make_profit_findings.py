@@ -3,7 +3,7 @@ profit experiment of Section 5.2 (first 200 replications of the profit-
 experiment workload), next to which Table 1's ISJL rows do not hold.
 
 FCFS and LJF reproduce Table 1 within the five-replication sampling noise;
-ISJL (Algorithm 2 under this build's readings) is slower than LJF here, while
+ISJL (Algorithm 2 under the simulator's readings) is slower than LJF here, while
 Table 1 reports it 3.5% to 22% faster.  The file records the oracle's means so
 the finding is pinned.  Only the oracle computes anything here.
 

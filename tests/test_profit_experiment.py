@@ -5,7 +5,7 @@ FCFS and LJF must reproduce Table 1 within the sampling noise of a
 five-replication mean (the paper averages five replications); this pins the
 workload recipe, the cost decomposition (Theorem "Profit decomposition") and
 both baselines to numbers the paper prints.  ISJL does not reproduce its
-Table 1 rows under this build's reading of Algorithm 2 (it is slower than LJF
+Table 1 rows under the simulator's reading of Algorithm 2 (it is slower than LJF
 on this workload, the table has it faster): the oracle's values are pinned in
 tests/golden/profit_isjl_oracle.txt and the gap is asserted, as a finding.
 """
