@@ -1254,17 +1254,27 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     __syncwarp();
 }
 
-// resident blocks per SM the register allocation is bounded for (measured
-// best on GB300 for the online sweep: 4 for both variants)
-#ifndef ISJL_SIM_MIN_BLOCKS_STEP
-#define ISJL_SIM_MIN_BLOCKS_STEP 4
+// resident blocks per SM the register allocation is bounded for, per
+// instantiation (measured on GB300): 4 (up to 128 registers) in general;
+// SPL_BLOCKS16 for 16 register rows (B > 256), where shared memory already
+// limits large instances to 2 blocks per SM and a tighter bound only spills;
+// SPL_BLOCKS4_STEP for the step kernel with 4 rows (B <= 128)
+#ifndef ISJL_SIM_MIN_BLOCKS
+#define ISJL_SIM_MIN_BLOCKS 4
 #endif
-#ifndef ISJL_SIM_MIN_BLOCKS_EPOCH
-#define ISJL_SIM_MIN_BLOCKS_EPOCH 4
+#ifndef ISJL_SIM_BLOCKS16
+#define ISJL_SIM_BLOCKS16 3
 #endif
+#ifndef ISJL_SIM_BLOCKS4_STEP
+#define ISJL_SIM_BLOCKS4_STEP 5
+#endif
+template <int SPL, bool EPOCH>
+constexpr int sim_min_blocks() {
+    return SPL >= 16 ? ISJL_SIM_BLOCKS16 : (SPL == 4 && !EPOCH ? ISJL_SIM_BLOCKS4_STEP : ISJL_SIM_MIN_BLOCKS);
+}
 
 template <int SPL, bool EPOCH>
-__global__ void __launch_bounds__(kSimWarpsPerBlock * 32, EPOCH ? ISJL_SIM_MIN_BLOCKS_EPOCH : ISJL_SIM_MIN_BLOCKS_STEP)
+__global__ void __launch_bounds__(kSimWarpsPerBlock * 32, sim_min_blocks<SPL, EPOCH>())
 sim_kernel(SimArgs A, int64_t n_tasks) {
     extern __shared__ __align__(16) int32_t smem[];
     const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
