@@ -76,3 +76,17 @@ def test_run_grids_are_valid():
     for wid, (pols, deltas, per_core) in bench.GRIDS.items():
         assert wid in W.WORKLOADS and len(pols) == len(deltas) <= 32 and per_core >= 1
         assert set(pols) <= {"fcfs", "ljf", "isjl", "sjf", "isjl_beta"}
+
+
+def test_epoch_count_counts_distinct_event_steps():
+    """The event-driven kernel's algorithmic work counts epochs: per (run,
+    instance), the distinct steps at which some request starts or completes;
+    -1 entries (requests that never started or finished) are not steps."""
+    import bench
+    start = np.array([[[0, 0, 3, -1], [5, 5, 5, 5]]], np.int32)          # 1 run, 2 instances, n = 4
+    compl = np.array([[[3, 4, 9, -1], [6, 7, 7, 8]]], np.int32)
+    # instance 0: {0, 3, 4, 9} -> 4; instance 1: {5, 6, 7, 8} -> 4
+    assert bench.epoch_count(start, compl) == 8
+    two = np.concatenate([start, start])
+    assert bench.epoch_count(two, np.concatenate([compl, compl])) == 16
+    assert bench.epoch_count(np.full((1, 1, 3), -1, np.int32), np.full((1, 1, 3), -1, np.int32)) == 0
