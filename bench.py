@@ -75,6 +75,10 @@ PROBE_LAUNCHES = 3
 # workload: 748.6 MB measured by ncu on the first 4,096 instances, scaled by
 # 10,000 / 4,096 (profiles/sim_kernel_step_online_delta_sweep_4096.md)
 SIM_DRAM_BYTES_PER_LAUNCH = 748.6e6 * 10_000 / 4_096
+# issue-slot and ALU-pipe utilisation of the same capture (smsp__issue_active and
+# sm__inst_executed_pipe_alu, percent of peak while active), reported beside the roofline
+SIM_NCU_ISSUE_ACTIVE = 0.718
+SIM_NCU_ALU_PIPE = 0.700
 
 
 def workload_config(kernel, wl, n_inst, policies, deltas, flush):
@@ -457,6 +461,9 @@ def main():
         roofline = roof("sim_kernel (epoch)", ops_epoch, sim_avg_ms, None)
     else:
         roofline = roof("sim_kernel (step)", ops_step, sim_avg_ms, SIM_DRAM_BYTES_PER_LAUNCH if full else None)
+        if full:
+            roofline["ncu_issue_active"] = SIM_NCU_ISSUE_ACTIVE
+            roofline["ncu_alu_pipe"] = SIM_NCU_ALU_PIPE
     if other is not None:
         o_ops = ops_epoch if other["kernel"] == "epoch" else ops_step
         o_roof = roof(f"sim_kernel ({other['kernel']})", o_ops, other["sim_ms_per_launch"], None)

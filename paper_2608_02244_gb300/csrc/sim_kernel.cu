@@ -35,7 +35,10 @@
 //   epoch kernel  jumps from event to event (arrival, completion, o_1's delay
 //                 expiry) and adds the cost of the L steps in between in closed
 //                 form; the running set is constant there and progress moves
-//                 in lockstep, so every counter is identical.
+//                 in lockstep, so every counter is identical.  While LJF has a
+//                 batch running or ISJL's gate is shut, completions that do not
+//                 change the running set's earliest or latest start are served
+//                 in the same pass (a completion window).
 // Admissions happen only at events: between events the running set, the KV
 // reservation and the queue are unchanged and A_max only grows, so a step
 // that could not start a request is followed by steps that cannot either.
