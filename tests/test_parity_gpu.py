@@ -368,6 +368,27 @@ def test_integer_rate_probe(S):
         assert 1e12 < rate < props.multi_processor_count * 128 * 2.2e9, (kind, rate)
 
 
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_completion_windows(S, O, epoch):
+    """Instances where the event-driven kernel serves long completion windows:
+    bursts of arrivals (many requests start at the same step), lengths from a
+    small set (ties in completion and in start), LJF batches and ISJL with a
+    gate shut for most of a stage (alpha 0, 2, 8, 64), with and without a KV
+    cap, and step guards that stop a run inside a window."""
+    rng = np.random.default_rng(33)
+    n = 300
+    a = np.sort(rng.choice(np.array([0, 0, 0, 40, 120, 121, 500], np.int32), (4, n)), axis=1).astype(np.int32)
+    p = rng.integers(0, 3, (4, n)).astype(np.int32)
+    o = rng.choice(np.array([1, 5, 5, 9, 30, 31, 200], np.int32), (4, n)).astype(np.int32)
+    pols = ["ljf", "isjl", "isjl", "isjl", "isjl", "isjl_beta", "fcfs"]
+    ds = [0, 0, 2, 8, 64, 8, 0]
+    for B in (8, 64):
+        for kv in (INF, 900):
+            run_both(S, O, a, p, o, B, pols, ds, kv, epoch)
+        for ms in (37, 401, 1500):
+            run_both(S, O, a, p, o, B, pols, ds, 900, epoch, max_steps=ms)
+
+
 def test_invalid_arguments_rejected(S):
     import torch
     sm = S.Simulator(1, 4, 2)
