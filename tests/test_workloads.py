@@ -35,3 +35,4 @@ def test_ranges():
     assert (np.diff(a, axis=1) >= 0).all() and p.min() >= 16 and p.max() <= 32768 and o.max() <= 16384
     # mean gap 0.05: 1e5 requests arrive within a few thousand steps
     assert 4000 < a[0, -1] < 6000
+
