@@ -389,6 +389,42 @@ def test_completion_windows(S, O, epoch):
             run_both(S, O, a, p, o, B, pols, ds, 900, epoch, max_steps=ms)
 
 
+@pytest.mark.parametrize("epoch", EPOCHS)
+def test_random_configurations(S, O, epoch):
+    """Randomised shapes against the oracle, every policy: request counts
+    from 1 to 300 (ragged counts on some), B from 1 to 512 (every register
+    row count), budgets from 0 to infinity, KV caps from the largest request
+    upwards or none, arrivals offline, spread or in bursts, lengths with many
+    ties or spread out, upper-bound slack on some, step guards on some."""
+    rng = np.random.default_rng(2024)
+    pols = ["fcfs", "ljf", "sjf", "isjl", "isjl", "isjl", "isjl_beta"]
+    for case in range(60):
+        n_inst = int(rng.integers(1, 5))
+        n = int(rng.choice([1, 2, 7, 33, 64, 150, 300]))
+        B = int(rng.choice([1, 2, 3, 31, 32, 33, 64, 100, 128, 129, 256, 257, 384, 512]))
+        kind = case % 3
+        if kind == 0:
+            a = np.zeros((n_inst, n), np.int32)
+        elif kind == 1:
+            a = np.sort(rng.integers(0, 5 * n + 1, (n_inst, n)), axis=1).astype(np.int32)
+        else:
+            a = np.sort(rng.choice(np.array([0, 3, 3, 50, 51, 400]), (n_inst, n)), axis=1).astype(np.int32)
+        if case % 2:
+            o = rng.choice(np.array([1, 4, 4, 9, 16, 16, 70]), (n_inst, n)).astype(np.int32)
+        else:
+            o = rng.integers(1, 400, (n_inst, n)).astype(np.int32)
+        p = rng.integers(0, 3, (n_inst, n)).astype(np.int32)      # o_i = prompt + output >= 1
+        o = np.where(p + np.maximum(o - p, 0) < 1, 1, np.maximum(o - p, 0)).astype(np.int32)
+        big = int((p + o).max())
+        e = rng.integers(0, 20, (n_inst, n)).astype(np.int32) if case % 4 == 3 else None
+        big_u = big + (int(e.max()) if e is not None else 0)
+        kv = INF if case % 5 == 0 else int(rng.integers(big_u, big_u * 6 + 2))
+        ds = [0, 0, 0, 0, int(rng.integers(1, 40)), INF, int(rng.integers(1, 40))]
+        counts = rng.integers(0, n + 1, n_inst).astype(np.int32) if case % 6 == 5 else None
+        ms = int(rng.integers(1, 3 * n + 5)) if case % 7 == 6 else 0
+        run_both(S, O, a, p, o, B, pols, ds, kv, epoch, counts=counts, slack=e, max_steps=ms)
+
+
 def test_invalid_arguments_rejected(S):
     import torch
     sm = S.Simulator(1, 4, 2)
