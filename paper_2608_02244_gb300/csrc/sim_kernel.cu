@@ -154,6 +154,15 @@ __device__ __forceinline__ void mad_wide(int64_t &acc, uint32_t a, uint32_t b) {
     asm("mad.wide.u32 %0, %1, %2, %0;" : "+l"(acc) : "r"(a), "r"(b));
 }
 
+// warp sum of a 64-bit value (modulo 2^64) by three independent 32-bit warp
+// reductions of its 22-, 22- and 20-bit pieces (each piece's sum is below 2^27)
+__device__ __forceinline__ uint64_t warp_sum_u64(uint64_t v) {
+    const uint32_t a = __reduce_add_sync(kFull, (uint32_t)v & 0x3FFFFFu);
+    const uint32_t b = __reduce_add_sync(kFull, (uint32_t)(v >> 22) & 0x3FFFFFu);
+    const uint32_t c = __reduce_add_sync(kFull, (uint32_t)(v >> 44));
+    return (uint64_t)a + ((uint64_t)b << 22) + ((uint64_t)c << 44);
+}
+
 __device__ __forceinline__ int64_t warp_sum64(int64_t v) {
 #pragma unroll
     for (int s = 16; s > 0; s >>= 1) v += __shfl_xor_sync(kFull, v, s);
@@ -1080,23 +1089,25 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         // and the extent smax - smin is constant.  Requests with c_i < K
         // complete inside the window and leave here.
         auto window = [&](int32_t K) {
-            const int64_t m0 = (int64_t)k - smin + 1;
-            int64_t wl = 0, el = 0, cl = 0, sl = 0;
+            // twice the W term per slot: L_i (2 m0 - 1 + L_i), m0 = k - smin + 1;
+            // all factors below 2^32
+            const uint32_t m2 = 2u * (uint32_t)(k - smin) + 1u;
+            uint64_t wl2 = 0, el = 0, cl = 0, sl = 0;
             int32_t tl = 0, cmx = 0, nf = 0, of = 0;
             uint32_t fm = 0u;
 #pragma unroll
             for (int r = 0; r < SPL; ++r)
                 if (busy >> r & 1u) {
                     const int32_t c = sc[r];
-                    const int64_t Li = (int64_t)min(c, K) - k;
-                    wl += Li * m0 + Li * (Li - 1) / 2;
-                    el += Li * (int64_t)(sa[r] - smin);
+                    const uint32_t Li = (uint32_t)(min(c, K) - k);
+                    wl2 += (uint64_t)Li * (m2 + Li);
+                    el += (uint64_t)Li * (uint32_t)(sa[r] - smin);
                     tl += (int32_t)Li;
                     if (c < K) {                                  // completes inside the window
                         const int w = (r << 5) + lane;
                         fm |= 1u << r;
-                        cl += c;
-                        sl += sa[r];
+                        cl += (uint32_t)c;
+                        sl += (uint32_t)sa[r];
                         cmx = max(cmx, c);
                         nf++;
                         of += S.sres[w];
@@ -1106,13 +1117,13 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 }
             busy &= ~fm;
             recompute_lane();
-            W += warp_sum64(wl);
-            E += warp_sum64(el);
+            W += (int64_t)(warp_sum_u64(wl2) >> 1);             // every slot's term is even
+            E += (int64_t)warp_sum_u64(el);
             tok += (int32_t)__reduce_add_sync(kFull, (unsigned)tl);
             nf = (int32_t)__reduce_add_sync(kFull, (unsigned)nf);
             of = (int32_t)__reduce_add_sync(kFull, (unsigned)of);
-            sumc += warp_sum64(cl);
-            sum_st -= warp_sum64(sl);
+            sumc += (int64_t)warp_sum_u64(cl);
+            sum_st -= (int64_t)warp_sum_u64(sl);
             const int32_t cm = (int32_t)__reduce_max_sync(kFull, (unsigned)cmx);
             if (nf > 0) Tmake = max(Tmake, cm);
             done += nf;
@@ -1201,13 +1212,16 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     }
                 }
                 if (run_cnt > 0) {
-                    const int64_t L = nxt - k, s = run_cnt;
-                    const int64_t m0 = (int64_t)k - smin + 1;       // max r at step k
-                    const int32_t ext = smax - smin;                // max r - min r
-                    const int64_t sr = s * ((int64_t)k + 1) - sum_st;   // sum r at step k
-                    W += s * (L * m0 + L * (L - 1) / 2);
-                    E += L * (s * m0 - sr);
-                    sumext += L * ext;
+                    // L steps, max r = m0 + t at step k + t, sum r = s m0 - sum (s_i - smin) + s t:
+                    //   W += s (L m0 + L (L - 1) / 2) = s L (2 m0 + L - 1) / 2
+                    //   E += L sum (s_i - smin) = L (sum_st - s smin)
+                    const uint32_t L = (uint32_t)(nxt - k), s = (uint32_t)run_cnt;
+                    const uint32_t m0 = (uint32_t)(k - smin + 1);     // max r at step k
+                    const int32_t ext = smax - smin;                  // max r - min r
+                    const uint64_t wl = ((uint64_t)L * (2u * m0 + L - 1u)) >> 1;   // both factors < 2^32
+                    W += (int64_t)(wl * s);
+                    E += (int64_t)L * (sum_st - (int64_t)s * smin);
+                    mad_wide(sumext, L, (uint32_t)ext);
                     maxext = max(maxext, ext);
                     viol += ext > alpha32 ? (int32_t)L : 0;
                     kvviol += kv_over ? (int32_t)L : 0;
