@@ -48,6 +48,7 @@
 // start at a time.
 #include <climits>
 #include <cstdint>
+#include <type_traits>
 
 #include "sim_internal.cuh"
 
@@ -280,6 +281,11 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     const int64_t alpha = A.runs.delta[run];
     const int64_t beta = A.runs.beta[run];
     const int64_t kv_cap = A.kv_cap;
+    // reserved KV: at most B <= 512 running requests of length <= 65535, so
+    // below 2^25; the event-driven kernel keeps it in 32 bits (against the cap
+    // clamped to INT_MAX, which compares the same)
+    using kv_t = std::conditional_t<EPOCH, int32_t, int64_t>;
+    const kv_t kv_lim = EPOCH ? (kv_t)min(kv_cap, (int64_t)INT_MAX) : (kv_t)kv_cap;
     const int32_t *__restrict__ arr = A.arrival + base;
     const int32_t *__restrict__ oarr = A.o + base;              // planning lengths (u_i)
     const int32_t *__restrict__ otru = A.otrue ? A.otrue + base : nullptr;   // true lengths
@@ -314,7 +320,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     // o (o + 1) / 2 when a request starts and takes back the unserved part of
     // requests still running if a run stops early (the decomposition W = Q + E
     // of Section 5)
-    int64_t W = 0, R = 0, E = 0, sumc = 0, sumext = 0, peakkv = 0;
+    int64_t W = 0, R = 0, E = 0, sumc = 0, sumext = 0;
+    kv_t peakkv = 0;
     int32_t Tb = 0, tok = 0, maxext = 0, viol = 0, peakb = 0, Tmake = 0, kvviol = 0;
 
     if (status == ISJL_OK && n > 0) {
@@ -343,7 +350,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         // step kernel: A_max at the current step, from the last step's max reduction
         int32_t amax_c = 0;
         bool amax_ok = false;
-        int64_t kv_sum = 0, sum_st = 0;
+        kv_t kv_sum = 0;
+        int64_t sum_st = 0;
         // the next 32 unreleased requests (from win_base): arrival and sorted position, per lane
         int32_t win_base = 0, win_a = INT_MAX, win_p = 0;
         auto load_window = [&]() {
@@ -383,7 +391,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             cmin = min(cmin, k + oc);
             peakkv = max(peakkv, kv_sum);
             peakb = max(peakb, run_cnt);
-            kv_over = kv_sum > kv_cap;
+            kv_over = kv_sum > kv_lim;
             if (EPOCH) { sum_st += k; smin = min(smin, k); smax = k; }
             if (!EPOCH) mad_wide(R, ((uint32_t)oc * (uint32_t)(oc + 1)) >> 1, 1u);   // oc (oc + 1) < 2^32
             const int owner = w & 31, row = w >> 5;
@@ -404,7 +412,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         // warp-wide totals of c starts at step k made lane-parallel: kv_add their
         // reserved KV, my_cmin / rsum this lane's earliest completion and sum of
         // o (o + 1) / 2, top the highest row that received one, plus one
-        auto commit_starts = [&](int c, int64_t kv_add, int32_t my_cmin, uint64_t rsum, int top) {
+        auto commit_starts = [&](int c, kv_t kv_add, int32_t my_cmin, uint64_t rsum, int top) {
             __syncwarp();
             lane_cmin = min(lane_cmin, my_cmin);
             if (EPOCH && my_cmin != INT_MAX) { lane_smin = min(lane_smin, k); lane_smax = max(lane_smax, k); }
@@ -414,7 +422,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             cmin = min(cmin, (int32_t)__reduce_min_sync(kFull, (unsigned)my_cmin));
             peakkv = max(peakkv, kv_sum);
             peakb = max(peakb, run_cnt);
-            kv_over = kv_sum > kv_cap;
+            kv_over = kv_sum > kv_lim;
             if (EPOCH) { sum_st += (int64_t)c * k; smin = min(smin, k); smax = k; }
             if (!EPOCH) {
                 // rsum < 2^35 per lane: its low 24 bits and the rest summed by two reductions
@@ -439,7 +447,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (lane >= d) pre += t;
             }
             const int nfree = (int)__reduce_add_sync(kFull, (unsigned)__popc(fm));
-            const bool fit = lane < m && lane < nfree && kv_sum + pre <= kv_cap;
+            const bool fit = lane < m && lane < nfree && kv_sum + pre <= kv_lim;
             const int c = __popc(__ballot_sync(kFull, fit));
             if (c == 0) return 0;
             const int oc_l = (otru && lane < c) ? otru[ce] : co;  // it finishes after its true length
@@ -509,7 +517,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             run_cnt -= nf;
             if (!EPOCH && nf > 0) amax_ok = false;
             kv_sum -= of;
-            kv_over = kv_sum > kv_cap;
+            kv_over = kv_sum > kv_lim;
             sumc += (int64_t)nf * c;
             Tmake = c;
             cmin = __reduce_min_sync(kFull, lane_cmin);
@@ -629,7 +637,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (w < 0) return;
                 const int p = head();
                 if (p >= n) { broken = true; return; }
-                if (kv_sum + ho > kv_cap) return;
+                if (kv_sum + ho > kv_lim) return;
                 if (nseq < 2) {
                     const int e = he, oe = ho;
                     pop_head(p);
@@ -659,7 +667,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         auto plan_bulk = [&](uint32_t cand, bool over) -> bool {
             bool stopped = false;
             int c = 0, top = 0;
-            int64_t kv_add = 0;
+            kv_t kv_add = 0;
             int32_t my_cmin = INT_MAX;
             uint64_t rsum = 0;
 #pragma unroll
@@ -680,7 +688,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         const int t = __shfl_up_sync(kFull, pre, d);
                         if (lane >= d) pre += t;
                     }
-                    const bool fits = el && kv_sum + kv_add + pre <= kv_cap;
+                    const bool fits = el && kv_sum + kv_add + pre <= kv_lim;
                     const unsigned fb = __ballot_sync(kFull, fits);
                     if (fb != __ballot_sync(kFull, el)) stopped = true;   // the first one that does not fit
                     if (fits) {
@@ -703,7 +711,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     }
                     if (fb) top = r + 1;
                     c += __popc(fb);
-                    kv_add += (int64_t)__reduce_add_sync(kFull, fits ? (unsigned)oe : 0u);
+                    kv_add += (kv_t)__reduce_add_sync(kFull, fits ? (unsigned)oe : 0u);
                 }
             }
             if (c > 0) commit_starts(c, kv_add, my_cmin, rsum, top);
@@ -883,7 +891,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     if (run_cnt >= B) { blocked = true; break; }
                     if (fcfs >= rel) break;
                     if (fo < 0) fo = oarr[fcfs];
-                    if (kv_sum + fo > kv_cap) { blocked = true; break; }
+                    if (kv_sum + fo > kv_lim) { blocked = true; break; }
                     if (nseq < 2) {
                         const int w = lowest_worker(vmask & ~busy, lane);
                         if (w < 0) { broken = true; return; }
@@ -910,7 +918,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     const int hi = bs_last(S, words1, lane);
                     if (hi < 0 || hi >= n) { broken = true; return; }
                     const int omin = osrt[hi];
-                    if (kv_sum + omin > kv_cap) break;
+                    if (kv_sum + omin > kv_lim) break;
                     const int g = first_pos_le(osrt, n, omin, lane);
                     if (nseq < 2) {
                         const int p = bs_next(S, words0, words1, g, lane);
@@ -972,7 +980,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         }
                         if (w >= 1 && w < nlong && e == S.slong[w] && !L1_started) continue;  // o_j after o_1
                         const int oe = S.spsum[w];                 // o of the worker's next entry
-                        if (kv_sum + oe > kv_cap) { stop = true; break; }
+                        if (kv_sum + oe > kv_lim) { stop = true; break; }
                         const int nx = pnext[e];
                         __syncwarp();
                         if (lane == 0) {
@@ -1129,7 +1137,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             done += nf;
             run_cnt -= nf;
             kv_sum -= of;
-            kv_over = kv_sum > kv_cap;
+            kv_over = kv_sum > kv_lim;
             cmin = __reduce_min_sync(kFull, lane_cmin);
             const int32_t ext = smax - smin;                  // unchanged inside the window
             const int32_t L = K - k;
@@ -1187,7 +1195,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         } else {
             // --------------------------------------------------- epoch kernel
             for (;;) {
-                if ((int64_t)k > max_steps) { status = ISJL_ERR_STEP_LIMIT; break; }
+                if (k >= step_guard) { status = ISJL_ERR_STEP_LIMIT; break; }   // k > max_steps
                 if (k >= next_arr) release();
                 if (k == cmin) retire(k);
                 if (done == n) break;
@@ -1203,7 +1211,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 // before the running set's earliest or latest start changes, so
                 // completions in between end no epoch of their own
                 if (run_cnt > 0 && !kv_over && nxt == cmin &&
-                    (policy == ISJL_POLICY_LJF || (policy == ISJL_POLICY_ISJL && (int64_t)k - smin > alpha))) {
+                    (policy == ISJL_POLICY_LJF || (policy == ISJL_POLICY_ISJL && k - smin > alpha32))) {
                     const int32_t K = min(window_end(), step_guard);
                     if (K > nxt) {
                         window(K);
