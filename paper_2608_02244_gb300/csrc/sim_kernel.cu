@@ -48,7 +48,6 @@
 // start at a time.
 #include <climits>
 #include <cstdint>
-#include <type_traits>
 
 #include "sim_internal.cuh"
 
@@ -282,10 +281,9 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     const int64_t beta = A.runs.beta[run];
     const int64_t kv_cap = A.kv_cap;
     // reserved KV: at most B <= 512 running requests of length <= 65535, so
-    // below 2^25; the event-driven kernel keeps it in 32 bits (against the cap
-    // clamped to INT_MAX, which compares the same)
-    using kv_t = std::conditional_t<EPOCH, int32_t, int64_t>;
-    const kv_t kv_lim = EPOCH ? (kv_t)min(kv_cap, (int64_t)INT_MAX) : (kv_t)kv_cap;
+    // below 2^25; kept in 32 bits, against the cap clamped to INT_MAX (which
+    // compares the same)
+    const int32_t kv_lim = (int32_t)min(kv_cap, (int64_t)INT_MAX);
     const int32_t *__restrict__ arr = A.arrival + base;
     const int32_t *__restrict__ oarr = A.o + base;              // planning lengths (u_i)
     const int32_t *__restrict__ otru = A.otrue ? A.otrue + base : nullptr;   // true lengths
@@ -321,7 +319,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
     // requests still running if a run stops early (the decomposition W = Q + E
     // of Section 5)
     int64_t W = 0, R = 0, E = 0, sumc = 0, sumext = 0;
-    kv_t peakkv = 0;
+    int32_t peakkv = 0;
     int32_t Tb = 0, tok = 0, maxext = 0, viol = 0, peakb = 0, Tmake = 0, kvviol = 0;
 
     if (status == ISJL_OK && n > 0) {
@@ -350,8 +348,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         // step kernel: A_max at the current step, from the last step's max reduction
         int32_t amax_c = 0;
         bool amax_ok = false;
-        kv_t kv_sum = 0;
-        int64_t sum_st = 0;
+        int32_t kv_sum = 0;
+        uint32_t sum_st = 0;   // epoch kernel: the running requests' start steps, summed modulo 2^32
         // the next 32 unreleased requests (from win_base): arrival and sorted position, per lane
         int32_t win_base = 0, win_a = INT_MAX, win_p = 0;
         auto load_window = [&]() {
@@ -392,7 +390,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             peakkv = max(peakkv, kv_sum);
             peakb = max(peakb, run_cnt);
             kv_over = kv_sum > kv_lim;
-            if (EPOCH) { sum_st += k; smin = min(smin, k); smax = k; }
+            if (EPOCH) { sum_st += (uint32_t)k; smin = min(smin, k); smax = k; }
             if (!EPOCH) mad_wide(R, ((uint32_t)oc * (uint32_t)(oc + 1)) >> 1, 1u);   // oc (oc + 1) < 2^32
             const int owner = w & 31, row = w >> 5;
             if (!EPOCH && row >= adv_rows) adv_rows = row_class<SPL>(row + 1);
@@ -412,7 +410,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         // warp-wide totals of c starts at step k made lane-parallel: kv_add their
         // reserved KV, my_cmin / rsum this lane's earliest completion and sum of
         // o (o + 1) / 2, top the highest row that received one, plus one
-        auto commit_starts = [&](int c, kv_t kv_add, int32_t my_cmin, uint64_t rsum, int top) {
+        auto commit_starts = [&](int c, int32_t kv_add, int32_t my_cmin, uint64_t rsum, int top) {
             __syncwarp();
             lane_cmin = min(lane_cmin, my_cmin);
             if (EPOCH && my_cmin != INT_MAX) { lane_smin = min(lane_smin, k); lane_smax = max(lane_smax, k); }
@@ -423,7 +421,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             peakkv = max(peakkv, kv_sum);
             peakb = max(peakb, run_cnt);
             kv_over = kv_sum > kv_lim;
-            if (EPOCH) { sum_st += (int64_t)c * k; smin = min(smin, k); smax = k; }
+            if (EPOCH) { sum_st += (uint32_t)c * (uint32_t)k; smin = min(smin, k); smax = k; }
             if (!EPOCH) {
                 // rsum < 2^35 per lane: its low 24 bits and the rest summed by two reductions
                 const unsigned lo = __reduce_add_sync(kFull, (unsigned)(rsum & 0xFFFFFFu));
@@ -512,7 +510,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             nf = (int)__reduce_add_sync(kFull, (unsigned)nf);
             of = (int)__reduce_add_sync(kFull, (unsigned)of);
             if (EPOCH)   // starts are within 65535 steps of c, so the offsets fit 32 bits
-                sum_st -= (int64_t)__reduce_add_sync(kFull, sf) + (int64_t)nf * (c - 65536);
+                sum_st -= __reduce_add_sync(kFull, sf) + (uint32_t)nf * (uint32_t)(c - 65536);
             done += nf;
             run_cnt -= nf;
             if (!EPOCH && nf > 0) amax_ok = false;
@@ -527,9 +525,9 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             }
         };
         // A_max(k): largest progress among running requests (0 if none)
-        auto amax_now = [&]() -> int64_t {
+        auto amax_now = [&]() -> int32_t {
             if (run_cnt == 0) return 0;
-            if (EPOCH) return (int64_t)k - smin;
+            if (EPOCH) return k - smin;
             if (!amax_ok) {
                 if constexpr (kPacked) {
                     uint32_t m = 0u;    // packed progress: the larger value has the larger a
@@ -667,7 +665,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
         auto plan_bulk = [&](uint32_t cand, bool over) -> bool {
             bool stopped = false;
             int c = 0, top = 0;
-            kv_t kv_add = 0;
+            int32_t kv_add = 0;
             int32_t my_cmin = INT_MAX;
             uint64_t rsum = 0;
 #pragma unroll
@@ -711,7 +709,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     }
                     if (fb) top = r + 1;
                     c += __popc(fb);
-                    kv_add += (kv_t)__reduce_add_sync(kFull, fits ? (unsigned)oe : 0u);
+                    kv_add += (int32_t)__reduce_add_sync(kFull, fits ? (unsigned)oe : 0u);
                 }
             }
             if (c > 0) commit_starts(c, kv_add, my_cmin, rsum, top);
@@ -952,20 +950,20 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 const bool nothing_runs = run_cnt == 0;
                 if (nothing_runs && plan_left == 0 && pend > 0) phase_one();
                 if (broken) return;
-                bool stop = amax_now() > alpha;                  // the gate A_max(k) <= alpha
+                bool stop = amax_now() > alpha32;                // the gate A_max(k) <= alpha
                 if (!stop && plan_left > 0) {
                     // plan starts, workers in order; entries that must wait (o_1's
                     // delay, o_j before o_1) are filtered out up front
                     uint32_t cand = resv & ~busy;
                     if (!L1_started) {
                         cand &= ~lhead;
-                        const bool over = (int64_t)k >= (int64_t)t0 + d1;
+                        const bool over = k >= t0 + d1;
                         if (!over && lane == 0) cand &= ~1u;        // worker 0 holds o_1
                     }
                     for (int nseq = 0;;) {
                         if (nseq >= 2) {                            // the rest at once
                             if (__ballot_sync(kFull, cand != 0u)) {
-                                const bool over = (int64_t)k >= (int64_t)t0 + d1;
+                                const bool over = k >= t0 + d1;
                                 stop = plan_bulk(cand, over);
                             }
                             break;
@@ -975,7 +973,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                         if (lane == (w & 31)) cand &= ~(1u << (w >> 5));
                         const int e = S.shead[w];
                         if (w == 0 && e == L1) {
-                            const bool over = (int64_t)k >= (int64_t)t0 + d1;
+                            const bool over = k >= t0 + d1;
                             if (!over) continue;                 // o_1 still delayed
                         }
                         if (w >= 1 && w < nlong && e == S.slong[w] && !L1_started) continue;  // o_j after o_1
@@ -1029,7 +1027,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 #pragma unroll
                 for (int r = 0; r < NR; ++r)
                     if (!(busy >> r & 1u)) sa[r] = L;
-                uint32_t last_mx = 0u;
+                uint32_t last_mx = 0u, smx = 0u, sext = 0u;   // sums over the stretch: L, r < 2^16
 #pragma unroll kUnroll
                 for (int j = 0; j < L; ++j) {
                     uint32_t m = 0u;
@@ -1042,15 +1040,18 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     const uint32_t mx = __reduce_max_sync(kFull, m) >> 16;          // max r
                     const uint32_t lo = __reduce_max_sync(kFull, m & 0xFFFFu);      // 65535 - min r
                     const int ext = (int)(mx + lo) - 65535;
-                    mad_wide(W, cnt, mx);                // |S| max r
-                    mad_wide(sumext, (uint32_t)ext, 1u);
+                    smx += mx;
+                    sext += (uint32_t)ext;
                     maxext = max(maxext, ext);
                     viol += ext > alpha32;
                     last_mx = mx;
                 }
+                mad_wide(W, cnt, smx);                   // |S| max r, summed over the steps
+                sumext += sext;
                 amax_c = (int32_t)last_mx;               // max progress entering step k + L
             } else {
                 int last_mx = 0;
+                uint32_t smx = 0u, sext = 0u;            // sums over the stretch: L, r < 2^16
 #pragma unroll kUnroll
                 for (int j = 0; j < L; ++j) {
                     int mx = INT_MIN;
@@ -1065,12 +1066,14 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                     mx = __reduce_max_sync(kFull, mx);
                     mn = __reduce_min_sync(kFull, mn);
                     const int ext = mx - (int)mn;
-                    mad_wide(W, cnt, (uint32_t)mx);      // |S| max r
-                    mad_wide(sumext, (uint32_t)ext, 1u);
+                    smx += (uint32_t)mx;
+                    sext += (uint32_t)ext;
                     maxext = max(maxext, ext);
                     viol += ext > alpha32;
                     last_mx = mx;
                 }
+                mad_wide(W, cnt, smx);                   // |S| max r, summed over the steps
+                sumext += sext;
                 amax_c = last_mx;                        // max progress entering step k + L
             }
             amax_ok = true;
@@ -1100,7 +1103,8 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             // twice the W term per slot: L_i (2 m0 - 1 + L_i), m0 = k - smin + 1;
             // all factors below 2^32
             const uint32_t m2 = 2u * (uint32_t)(k - smin) + 1u;
-            uint64_t wl2 = 0, el = 0, cl = 0, sl = 0;
+            uint64_t wl2 = 0, el = 0, cl = 0;
+            uint32_t sl = 0;
             int32_t tl = 0, cmx = 0, nf = 0, of = 0;
             uint32_t fm = 0u;
 #pragma unroll
@@ -1131,7 +1135,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             nf = (int32_t)__reduce_add_sync(kFull, (unsigned)nf);
             of = (int32_t)__reduce_add_sync(kFull, (unsigned)of);
             sumc += (int64_t)warp_sum_u64(cl);
-            sum_st -= (int64_t)warp_sum_u64(sl);
+            sum_st -= __reduce_add_sync(kFull, sl);
             const int32_t cm = (int32_t)__reduce_max_sync(kFull, (unsigned)cmx);
             if (nf > 0) Tmake = max(Tmake, cm);
             done += nf;
@@ -1221,14 +1225,16 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 }
                 if (run_cnt > 0) {
                     // L steps, max r = m0 + t at step k + t, sum r = s m0 - sum (s_i - smin) + s t:
-                    //   W += s (L m0 + L (L - 1) / 2) = s L (2 m0 + L - 1) / 2
-                    //   E += L sum (s_i - smin) = L (sum_st - s smin)
+                    //   W += s (L m0 + L (L - 1) / 2),  E += L sum (s_i - smin)
+                    // The epoch ends by the completion of the request that started at
+                    // smin, so max r <= its o <= 65535 throughout: the sum of max r over
+                    // the L <= 65535 steps fits 32 bits, and sum (s_i - smin) <
+                    // B * 65536 is exact from the modular sum of starts.
                     const uint32_t L = (uint32_t)(nxt - k), s = (uint32_t)run_cnt;
                     const uint32_t m0 = (uint32_t)(k - smin + 1);     // max r at step k
                     const int32_t ext = smax - smin;                  // max r - min r
-                    const uint64_t wl = ((uint64_t)L * (2u * m0 + L - 1u)) >> 1;   // both factors < 2^32
-                    W += (int64_t)(wl * s);
-                    E += (int64_t)L * (sum_st - (int64_t)s * smin);
+                    mad_wide(W, s, L * m0 + ((L * (L - 1u)) >> 1));
+                    mad_wide(E, L, sum_st - s * (uint32_t)smin);
                     mad_wide(sumext, L, (uint32_t)ext);
                     maxext = max(maxext, ext);
                     viol += ext > alpha32 ? (int32_t)L : 0;
