@@ -66,7 +66,7 @@ struct WarpSmem {
     int32_t *shead;   // [B] next ISJL plan entry of worker w (kNone = none)
     int32_t *stail;   // [B] last plan entry of worker w
     int32_t *slong;   // [B] long request o_j planned on worker j (1 <= j < n_long)
-    int32_t *srem;    // [B] ISJL packing budget left on worker w (Phase ONE only)
+    int32_t *srem;    // [B] ISJL packing budget of worker w at a stage start (Phase ONE only)
     int32_t *spsum;   // [B] ISJL pack sum on worker w in Phase ONE, then the o of its next plan entry
     int32_t *sres;    // [B] KV reserved by the request running on worker w (its planning length)
     uint32_t *pend0;  // [words0] bit p: sorted position p is pending
@@ -790,9 +790,20 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             const int64_t o_last = __reduce_max_sync(kFull, olast_l);
             pend -= nl;
             const int64_t theta = min(2 * alpha, o1 - o_last + beta);
-            // first fit of the shorter requests, in sorted order
+            // first fit of the shorter requests, in sorted order.  Nothing runs
+            // at a stage start, so the slot registers sa[] are free: they hold
+            // the packing budgets left, worker r * 32 + lane in sa[r] (-1 for
+            // worker 1 and past B: never chosen), and are reset to idle below.
+#pragma unroll
+            for (int r = 0; r < SPL; ++r) {
+                const int w = (r << 5) + lane;
+                sa[r] = w < B ? S.srem[w] : -1;
+            }
+            // maxrem bounds the largest budget from above; it is recomputed only
+            // when a candidate no larger than it fits nowhere (budgets only shrink)
             int maxrem = -1;
-            for (int w = lane; w < B; w += 32) maxrem = max(maxrem, S.srem[w]);
+#pragma unroll
+            for (int r = 0; r < SPL; ++r) maxrem = max(maxrem, sa[r]);
             maxrem = __reduce_max_sync(kFull, maxrem);
             int q = -1;
             int64_t x_prev = -1;
@@ -800,7 +811,7 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
             for (;;) {
                 const int64_t x = min(theta, (int64_t)maxrem);
                 if (x < 1) break;
-                // candidates with o > x fit nowhere now or later (budgets only shrink)
+                // candidates with o > x fit nowhere now or later
                 if (x != x_prev) { pos_x = first_pos_le(osrt, n, x, lane); x_prev = x; }
                 q = bs_next(S, words0, words1, max(pos_x, q + 1), lane);
                 if (q >= n) break;
@@ -810,32 +821,38 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 #pragma unroll
                 for (int r = 0; r < SPL; ++r) {
                     const int w = (r << 5) + lane;
-                    const bool fits = w < B && S.srem[w] >= oe;
-                    if (fits && w >= nl && w < B) mA |= 1u << r;
-                    if (fits && w >= 1 && w < nl) mB |= 1u << r;
+                    const bool fits = sa[r] >= oe;
+                    if (fits && w >= nl) mA |= 1u << r;
+                    if (fits && w < nl) mB |= 1u << r;
                 }
                 int w = lowest_worker(mA, lane);                // workers M+1..B first
                 if (w < 0) w = highest_worker(mB, lane);        // then M, M-1, ..., 2
-                if (w < 0) { broken = true; return; }
-                const int remw = S.srem[w];                     // the chosen worker's budget before
+                if (w < 0) {                                    // it stays queued; the bound was stale
+                    int m = -1;
+#pragma unroll
+                    for (int r = 0; r < SPL; ++r) m = max(m, sa[r]);
+                    maxrem = __reduce_max_sync(kFull, m);
+                    continue;
+                }
+                {
+                    const int dec = lane == (w & 31) ? oe : 0;   // the chosen worker's budget shrinks
+#pragma unroll
+                    for (int r = 0; r < SPL; ++r) sa[r] -= r == (w >> 5) ? dec : 0;
+                }
                 __syncwarp();
                 if (lane == 0) {
                     const int tl = S.stail[w];
                     if (tl < 0) S.shead[w] = e; else pnext[tl] = e;
                     S.stail[w] = e;
                     pnext[e] = kNone;
-                    S.srem[w] = remw - oe;
                     S.spsum[w] += oe;
                 }
                 bs_clear(S, q, lane);   // includes __syncwarp
                 pend--;
                 plan_left++;
-                if (remw == maxrem) {                            // the largest budget may have shrunk
-                    maxrem = -1;
-                    for (int w2 = lane; w2 < B; w2 += 32) maxrem = max(maxrem, S.srem[w2]);
-                    maxrem = __reduce_max_sync(kFull, maxrem);
-                }
             }
+#pragma unroll
+            for (int r = 0; r < SPL; ++r) sa[r] = kIdle;
             // worker j (2..M) runs o_j after its pack
             for (int w = 1 + lane; w < nl; w += 32) {
                 const int e = S.slong[w];
