@@ -31,6 +31,15 @@
  *     policies plan with u_i = o_i + e_i (sorting, M, cap_j, packs, Phase TWO
  *     order, KV reservation of u_i); requests still finish after o_i tokens
  *     and the gate uses their true progress.  e = 0 is the clairvoyant case.
+ *
+ * Parity unpinned (nothing the paper fixes decides these parts; the tests check
+ * them only by invariants and hand-derived schedules):
+ *   - the KV cap: beyond "sum of reservations <= kv_cap at every step" and the
+ *     kv_cap = INT32_MAX reductions, the paper gives no value to compare with;
+ *   - ISJL at 0 < alpha < infinity with B >= 3 when a pack holds a request
+ *     longer than alpha, so that the gate can hold a plan entry back: pinned
+ *     only by hand-derived worked examples, and it misses the 3/4 bound of the
+ *     competitive-ratio theorem for Algorithm 2 on recorded tiny instances.
  */
 #include <stdint.h>
 #include <stdlib.h>

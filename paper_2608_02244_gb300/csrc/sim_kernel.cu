@@ -967,7 +967,9 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 const bool nothing_runs = run_cnt == 0;
                 if (nothing_runs && plan_left == 0 && pend > 0) phase_one();
                 if (broken) return;
-                bool stop = amax_now() > alpha32;                // the gate A_max(k) <= alpha
+                // the gate A_max(k) <= alpha; progress stays below o <= 65535, so a
+                // budget of at least 65535 never shuts it
+                bool stop = alpha32 < 65535 && amax_now() > alpha32;
                 if (!stop && plan_left > 0) {
                     // plan starts, workers in order; entries that must wait (o_1's
                     // delay, o_j before o_1) are filtered out up front
