@@ -68,3 +68,28 @@ def test_b2_isjl_with_optimal_beta_meets_its_bound():
         assert (rec["violations"] == 0).all()
         for i in range(len(o)):
             assert O.opt_makespan(a[i], o[i], 2, d) >= bound * rec["T_make"][i] - 1e-9, (d, i)
+
+
+def test_ljf_and_lpt_bounds_against_the_unconstrained_optimum():
+    """Theorem "Competitive Ratio of Algorithm LJF": T_OPT / T_LJF >= B / (2B - 1),
+    and Graham's bound for list scheduling longest first (the proposition the
+    proofs use for Phase TWO; ISJL at alpha = infinity is that rule):
+    T_OPT / T_ISJL(inf) >= 3B / (4B - 1); T_OPT without the fairness
+    constraint, every tiny instance, B = 2 and 3.  The LJF bound is attained by
+    o = (2, 1, 1) with B = 2: LJF needs 3 steps, the optimum 2."""
+    import numpy as np
+    from oracle import oracle as O
+    from paper_2608_02244_gb300 import workloads as W
+    a, p, out = W.generate(2)
+    o = p + out
+    for B in (2, 3):
+        ljf, _, _ = O.run("ljf", B, 0, INF, a, p, out, per_request=False)
+        lpt, _, _ = O.run("isjl", B, INF, INF, a, p, out, per_request=False)
+        for i in range(len(o)):
+            T = O.opt_makespan(a[i], o[i], B, INF)
+            assert T * (2 * B - 1) >= B * int(ljf["T_make"][i]), (B, i)
+            assert T * (4 * B - 1) >= 3 * B * int(lpt["T_make"][i]), (B, i)
+    z = np.zeros((1, 3), np.int32)
+    out3 = np.array([[2, 1, 1]], np.int32)
+    rec, _, _ = O.run("ljf", 2, 0, INF, z, z, out3, per_request=False)
+    assert int(rec["T_make"][0]) == 3 and O.opt_makespan(z[0], out3[0], 2, INF) == 2
