@@ -805,6 +805,10 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
 #pragma unroll
             for (int r = 0; r < SPL; ++r) maxrem = max(maxrem, sa[r]);
             maxrem = __reduce_max_sync(kFull, maxrem);
+            // this lane's rows whose worker takes no long request (M+1..B)
+            uint32_t rows_short = 0u;
+#pragma unroll
+            for (int r = 0; r < SPL; ++r) rows_short |= (uint32_t)((r << 5) + lane >= nl) << r;
             int q = -1;
             int64_t x_prev = -1;
             int pos_x = 0;                                      // first sorted position with o <= x_prev
@@ -817,16 +821,11 @@ __device__ __forceinline__ void run_task(const SimArgs &A, const WarpSmem &S, in
                 if (q >= n) break;
                 const int e = perm[q];
                 const int oe = osrt[q];
-                uint32_t mA = 0u, mB = 0u;
+                uint32_t fit = 0u;                              // rows whose budget takes it
 #pragma unroll
-                for (int r = 0; r < SPL; ++r) {
-                    const int w = (r << 5) + lane;
-                    const bool fits = sa[r] >= oe;
-                    if (fits && w >= nl) mA |= 1u << r;
-                    if (fits && w < nl) mB |= 1u << r;
-                }
-                int w = lowest_worker(mA, lane);                // workers M+1..B first
-                if (w < 0) w = highest_worker(mB, lane);        // then M, M-1, ..., 2
+                for (int r = 0; r < SPL; ++r) fit |= (uint32_t)(sa[r] >= oe) << r;
+                int w = lowest_worker(fit & rows_short, lane);  // workers M+1..B first
+                if (w < 0) w = highest_worker(fit & ~rows_short, lane);   // then M, M-1, ..., 2
                 if (w < 0) {                                    // it stays queued; the bound was stale
                     int m = -1;
 #pragma unroll
