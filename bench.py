@@ -72,13 +72,13 @@ OPS_PER_EPOCH = 14
 PROBE_ITERS = 20_000
 PROBE_LAUNCHES = 3
 # DRAM bytes (read + write) per launch of the step simulation kernel on the full
-# workload: 741.2 MB measured by ncu on the first 4,096 instances, scaled by
+# workload: 742.6 MB measured by ncu on the first 4,096 instances, scaled by
 # 10,000 / 4,096 (profiles/sim_kernel_step_online_delta_sweep_4096.md)
-SIM_DRAM_BYTES_PER_LAUNCH = 741.2e6 * 10_000 / 4_096
+SIM_DRAM_BYTES_PER_LAUNCH = 742.6e6 * 10_000 / 4_096
 # issue-slot and ALU-pipe utilisation of the same capture (smsp__issue_active and
 # sm__inst_executed_pipe_alu, percent of peak while active), reported beside the roofline
-SIM_NCU_ISSUE_ACTIVE = 0.752
-SIM_NCU_ALU_PIPE = 0.686
+SIM_NCU_ISSUE_ACTIVE = 0.750
+SIM_NCU_ALU_PIPE = 0.681
 
 
 def workload_config(kernel, wl, n_inst, policies, deltas, flush):
